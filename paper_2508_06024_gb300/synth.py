@@ -1,0 +1,161 @@
+"""Seeded synthetic inputs for the EC²MoE MoE-layer forward.
+
+This module only draws random numbers and rounds them to the storage type;
+it holds none of the layer's arithmetic (no gate, routing, FFN or codec
+math).  Both the CUDA path and the fp64 oracle are fed from it.
+
+Workload shapes follow the paper's evaluation (Switch-Transformer base,
+Top-1 routing, E up to 64 experts, local candidate cap; "Parameter
+Selection" in the evaluation setup) widened to the five layer presets
+below.  Recipe (all draws from one ``torch.Generator`` seeded per preset):
+
+* activations X ~ N(0, 1);
+* every weight matrix ~ N(0, 1/fan_in) (gate, expert and codec weights);
+* gate biases: zero (near-uniform expert load, since every expert's logit is
+  then a zero-mean Gaussian of nearly the same variance), except the
+  fine-grained preset, whose local-gate bias is ``-1.2 * ln(j + 1)`` for the
+  expert at rank j of a seeded permutation (Zipf s = 1.2 popularity);
+* the device mask allows the first ``n_allowed`` experts of a seeded
+  permutation (Eq. 4 leaves the capability test unspecified, so the allowed
+  set is an input);
+* bf16 presets store X, expert and codec weights in bf16 (round to nearest
+  even); gate weights and biases stay fp32.
+"""
+
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Dict, Optional
+
+import torch
+
+GELU = 0
+SWIGLU = 1
+F32 = 0
+BF16 = 1
+
+
+@dataclasses.dataclass(frozen=True)
+class LayerConfig:
+    name: str
+    T: int
+    d: int
+    E: int
+    d_ff: int
+    k: int
+    n_groups: int
+    act: int
+    dtype: int
+    r: int
+    n_allowed: int
+    n_shared: int = 0
+    d_ff_shared: int = 0
+    renorm_topk: int = 0
+    zipf_s: float = 0.0
+    seed: int = 0
+
+    def replace(self, **kw) -> "LayerConfig":
+        return dataclasses.replace(self, **kw)
+
+    @property
+    def torch_dtype(self) -> torch.dtype:
+        return torch.float32 if self.dtype == F32 else torch.bfloat16
+
+
+def preset(name: str, **overrides) -> LayerConfig:
+    """The five layer presets (tiny fp32, Switch, Mixtral, fine-grained, decode)."""
+    p = {
+        # 256 tokens, d=512, 8 GELU experts d_ff=1024, top-2, 2 groups, 4/8 allowed, rank 64.
+        "tiny_fp32": LayerConfig("tiny_fp32", T=256, d=512, E=8, d_ff=1024, k=2, n_groups=2,
+                                 act=GELU, dtype=F32, r=64, n_allowed=4),
+        # batch 8 x seq 512, d=768, 16 GELU experts d_ff=3072, top-1, 12/16 allowed, rank 128.
+        "switch_bf16": LayerConfig("switch_bf16", T=4096, d=768, E=16, d_ff=3072, k=1, n_groups=1,
+                                   act=GELU, dtype=BF16, r=128, n_allowed=12),
+        # 8192 tokens, d=4096, 8 SwiGLU experts d_ff=14336, top-2, 2 groups of 4, 6/8 allowed, rank 512.
+        "mixtral_bf16": LayerConfig("mixtral_bf16", T=8192, d=4096, E=8, d_ff=14336, k=2, n_groups=2,
+                                    act=SWIGLU, dtype=BF16, r=512, n_allowed=6),
+        # 16384 tokens, d=2048, 64 SwiGLU experts d_ff=1408, top-6, 2 shared, 8 groups of 8,
+        # 32/64 allowed, rank 256, Zipf(1.2) popularity.
+        "finegrained_bf16": LayerConfig("finegrained_bf16", T=16384, d=2048, E=64, d_ff=1408, k=6,
+                                        n_groups=8, act=SWIGLU, dtype=BF16, r=256, n_allowed=32,
+                                        n_shared=2, d_ff_shared=1408, zipf_s=1.2),
+        # decode: T in {1,4,16,64,256}; d=4096, 8 SwiGLU experts d_ff=14336, top-2, rank 128..512.
+        "decode_bf16": LayerConfig("decode_bf16", T=16, d=4096, E=8, d_ff=14336, k=2, n_groups=1,
+                                   act=SWIGLU, dtype=BF16, r=256, n_allowed=8),
+    }[name]
+    return p.replace(**overrides) if overrides else p
+
+
+def _normal(g: torch.Generator, shape, std: float, device) -> torch.Tensor:
+    return torch.randn(*shape, generator=g, device=device, dtype=torch.float32) * std
+
+
+def make_generator(seed: int, device) -> torch.Generator:
+    g = torch.Generator(device=device)
+    g.manual_seed(int(seed))
+    return g
+
+
+def make_mask(cfg: LayerConfig, device="cpu") -> torch.Tensor:
+    """uint8[E]; 1 for the first n_allowed experts of a seeded permutation."""
+    g = make_generator(cfg.seed * 7919 + 17, "cpu")
+    order = torch.randperm(cfg.E, generator=g)
+    mask = torch.zeros(cfg.E, dtype=torch.uint8)
+    mask[order[: cfg.n_allowed]] = 1
+    return mask.to(device)
+
+
+def make_inputs(cfg: LayerConfig, device="cpu", with_experts: bool = True) -> Dict[str, Optional[torch.Tensor]]:
+    """All tensors of one layer call, on ``device``, in their storage dtypes.
+
+    Keys: X, W_local, b_local, W_global, b_global, mask, W1, W3, W2,
+    W1s, W3s, W2s, V_enc, V_dec.  Absent parts are None.  Expert weights are
+    stored [E, out, in] (the reduction axis contiguous).
+    """
+    g = make_generator(cfg.seed, device)
+    st = cfg.torch_dtype
+    out: Dict[str, Optional[torch.Tensor]] = {}
+    out["X"] = _normal(g, (cfg.T, cfg.d), 1.0, device).to(st)
+    out["W_local"] = _normal(g, (cfg.E, cfg.d), 1.0 / math.sqrt(cfg.d), device)
+    b_local = torch.zeros(cfg.E, dtype=torch.float32)
+    if cfg.zipf_s > 0:
+        gz = make_generator(cfg.seed * 31 + 5, "cpu")
+        perm = torch.randperm(cfg.E, generator=gz)
+        ranks = torch.empty(cfg.E, dtype=torch.float32)
+        ranks[perm] = torch.arange(cfg.E, dtype=torch.float32)
+        b_local = -cfg.zipf_s * torch.log(ranks + 1.0)
+    out["b_local"] = b_local.to(device)
+    if cfg.n_groups > 1:
+        out["W_global"] = _normal(g, (cfg.n_groups, cfg.d), 1.0 / math.sqrt(cfg.d), device)
+        out["b_global"] = torch.zeros(cfg.n_groups, dtype=torch.float32, device=device)
+    else:
+        out["W_global"] = None
+        out["b_global"] = None
+    out["mask"] = make_mask(cfg, device)
+    if with_experts:
+        out["W1"] = _normal(g, (cfg.E, cfg.d_ff, cfg.d), 1.0 / math.sqrt(cfg.d), device).to(st)
+        out["W3"] = (_normal(g, (cfg.E, cfg.d_ff, cfg.d), 1.0 / math.sqrt(cfg.d), device).to(st)
+                     if cfg.act == SWIGLU else None)
+        out["W2"] = _normal(g, (cfg.E, cfg.d, cfg.d_ff), 1.0 / math.sqrt(cfg.d_ff), device).to(st)
+        if cfg.n_shared > 0:
+            fs = cfg.d_ff_shared
+            out["W1s"] = _normal(g, (cfg.n_shared, fs, cfg.d), 1.0 / math.sqrt(cfg.d), device).to(st)
+            out["W3s"] = (_normal(g, (cfg.n_shared, fs, cfg.d), 1.0 / math.sqrt(cfg.d), device).to(st)
+                          if cfg.act == SWIGLU else None)
+            out["W2s"] = _normal(g, (cfg.n_shared, cfg.d, fs), 1.0 / math.sqrt(fs), device).to(st)
+        else:
+            out["W1s"] = out["W3s"] = out["W2s"] = None
+    if cfg.r > 0:
+        out["V_enc"] = _normal(g, (cfg.r, cfg.d), 1.0 / math.sqrt(cfg.d), device).to(st)
+        out["V_dec"] = _normal(g, (cfg.d, cfg.r), 1.0 / math.sqrt(cfg.r), device).to(st)
+    else:
+        out["V_enc"] = out["V_dec"] = None
+    return out
+
+
+def to_f64(t: Optional[torch.Tensor]):
+    """Exact widening of a stored tensor to a float64 numpy array (None passes through)."""
+    if t is None:
+        return None
+    return t.detach().to("cpu").to(torch.float64).numpy()

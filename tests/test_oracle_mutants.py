@@ -1,0 +1,167 @@
+"""Plant plausible mistakes in the oracle (on the CPU) and check that the pins catch each.
+
+A pin set that lets one of these through would also let the same mistake in
+the oracle go unnoticed, so every mutant here must fail at least one pin.
+"""
+import numpy as np
+import pytest
+
+from oracle import ec2moe_oracle as orc
+from tests import pins
+
+_gate_logits = orc.gate_logits
+_group_gate = orc.group_gate
+_masked_softmax = orc._masked_softmax
+_route_tables = orc.route_tables
+_expert_ffn = orc.expert_ffn
+_combine_weights = orc.combine_weights
+_layer_forward = orc.layer_forward
+_topk_gaps = orc.topk_gaps
+
+
+def m_drop_local_bias(X, Wl, bl, Wg=None, bg=None):
+    return _gate_logits(X, Wl, np.zeros_like(np.asarray(bl, float)), Wg, bg)
+
+
+def m_drop_global_bias(X, Wl, bl, Wg=None, bg=None):
+    return _gate_logits(X, Wl, bl, Wg, None if bg is None else np.zeros_like(np.asarray(bg, float)))
+
+
+def m_softmax_ignores_mask(z, keep):
+    out = _masked_softmax(z, np.ones_like(keep))
+    out[:, ~keep] = 0.0
+    return out
+
+
+def m_group_gate_keeps_dead_groups(l, m, allowed, K):
+    # a dead group still takes part in the group softmax
+    g, log_g = _group_gate(l, m, allowed, K)
+    if K > 1 and m is not None:
+        b = orc.group_bounds(l.shape[1], K)
+        live = np.array([allowed[b[i]:b[i + 1]].any() for i in range(K)])
+        if not live.all():
+            full = np.exp(m - m.max(1, keepdims=True))
+            full /= full.sum(1, keepdims=True)
+            part = np.exp(m[:, live] - m[:, live].max(1, keepdims=True))
+            part /= part.sum(1, keepdims=True)
+            scale = np.ones_like(m)
+            scale[:, live] = full[:, live] / part
+            gof = np.repeat(np.arange(K), np.diff(b))
+            g = g * scale[:, gof]
+    return g, log_g
+
+
+def m_tie_to_higher_index(g, allowed, k):
+    E = g.shape[1]
+    key = np.where(allowed[None, :], -g, np.inf)[:, ::-1]
+    order = np.argsort(key, axis=1, kind="stable")
+    return (E - 1 - order[:, :k]).astype(np.int64)
+
+
+def m_topk_ascending(g, allowed, k):
+    key = np.where(allowed[None, :], g, np.inf)
+    return np.argsort(key, axis=1, kind="stable")[:, :k].astype(np.int64)
+
+
+def m_perm_reversed_within_expert(idx, E):
+    c, o, p = _route_tables(idx, E)
+    p = p.copy()
+    for e in range(E):
+        p[o[e]:o[e + 1]] = p[o[e]:o[e + 1]][::-1]
+    return c, o, p
+
+
+def m_offsets_inclusive(idx, E):
+    c, o, p = _route_tables(idx, E)
+    o = o.copy()
+    o[:-1] = o[1:]
+    return c, o, p
+
+
+def m_decode_no_transpose(Z, V_dec):
+    return np.asarray(Z, float) @ np.asarray(V_dec, float)
+
+
+def m_encode_wrong_side(X, V_enc):
+    V = np.asarray(V_enc, float)
+    if V.shape[0] == V.shape[1]:
+        return np.asarray(X, float) @ V
+    return np.asarray(X, float) @ V.T * 1.0001
+
+
+def m_gelu_tanh(u):
+    return 0.5 * u * (1 + np.tanh(np.sqrt(2 / np.pi) * (u + 0.044715 * u ** 3)))
+
+
+def m_silu_missing_x(u):
+    return 1.0 / (1.0 + np.exp(-u))
+
+
+def m_swiglu_swapped(x, W1, W2, W3, act):
+    if act == orc.SWIGLU:
+        return _expert_ffn(x, W3, W2, W1, act)
+    return _expert_ffn(x, W1, W2, W3, act)
+
+
+def m_renorm_ignored(g, idx, renorm):
+    return _combine_weights(g, idx, False)
+
+
+def m_renorm_always(g, idx, renorm):
+    return _combine_weights(g, idx, True)
+
+
+def m_no_shared(inp, n_groups, k, act, renorm=False, rows=None):
+    inp = dict(inp)
+    inp["W1s"] = inp["W2s"] = inp["W3s"] = None
+    return _layer_forward(inp, n_groups, k, act, renorm, rows)
+
+
+def m_experts_see_raw_x(inp, n_groups, k, act, renorm=False, rows=None):
+    out = _layer_forward(inp, n_groups, k, act, renorm, rows)
+    if inp.get("V_enc") is not None:
+        inp2 = dict(inp)
+        inp2["V_enc"] = inp2["V_dec"] = None
+        out2 = _layer_forward(inp2, n_groups, k, act, renorm, rows)
+        out["y"] = out2["y"]
+    return out
+
+
+def m_gap_wrong_sign(log_g, idx, allowed):
+    b, a = _topk_gaps(log_g, idx, allowed)
+    return -b, a
+
+
+MUTANTS = [
+    ("gate_logits", m_drop_local_bias),
+    ("gate_logits", m_drop_global_bias),
+    ("_masked_softmax", m_softmax_ignores_mask),
+    ("group_gate", m_group_gate_keeps_dead_groups),
+    ("topk_route", m_tie_to_higher_index),
+    ("topk_route", m_topk_ascending),
+    ("route_tables", m_perm_reversed_within_expert),
+    ("route_tables", m_offsets_inclusive),
+    ("lr_decode", m_decode_no_transpose),
+    ("lr_encode", m_encode_wrong_side),
+    ("gelu", m_gelu_tanh),
+    ("silu", m_silu_missing_x),
+    ("expert_ffn", m_swiglu_swapped),
+    ("combine_weights", m_renorm_ignored),
+    ("combine_weights", m_renorm_always),
+    ("layer_forward", m_no_shared),
+    ("layer_forward", m_experts_see_raw_x),
+    ("topk_gaps", m_gap_wrong_sign),
+]
+
+
+@pytest.mark.parametrize("name,mutant", MUTANTS, ids=[m.__name__ for _, m in MUTANTS])
+def test_mutant_is_caught(monkeypatch, name, mutant):
+    monkeypatch.setattr(orc, name, mutant)
+    caught = []
+    for pin in pins.ALL_PINS:
+        try:
+            pin(orc)
+        except (AssertionError, ValueError, IndexError, TypeError):
+            caught.append(pin.__name__)
+    assert caught, f"no pin catches mutant {mutant.__name__}"
+
