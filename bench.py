@@ -1,0 +1,444 @@
+#!/usr/bin/env python
+"""Throughput of the EC²MoE MoE-layer forward on GB300; prints one JSON line.
+
+A step is one ``ec2moe_layer_forward`` (mask -> group gate -> Top-k ->
+histogram/permute -> low-rank encode/decode -> grouped expert FFN ->
+gate-weighted combine) over one batch of synthetic tokens of the workload.
+Default workload: the Switch-style bf16 layer (4096 tokens = batch 8 x seq 512,
+d_model 768, 16 GELU experts with d_ff 3072, Top-1, 12 of 16 experts allowed,
+rank-128 codec).
+
+Timing: W untimed warm-up steps, then K steps, each bracketed by CUDA events
+on the launching stream with L2 flushed (256 MiB write) between steps; a
+barrier and a device synchronise bracket the timed loop; the max over ranks is
+reported.  Under torchrun each rank runs its own batch (token-parallel
+replicas, no collective on the data path; weak scaling).
+
+``--impl reference`` times the fp64 CPU oracle instead, on the host cores.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "MoE-layer tokens/s (gate→experts→combine + LR codec), % bf16 tensor peak"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="switch_bf16")
+    ap.add_argument("--T", type=int, default=0, help="override the token count (0 = preset)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU baseline sample")
+    return ap.parse_args()
+
+
+def workload_config(name: str, T: int = 0):
+    from paper_2508_06024_gb300 import synth as S
+    cfg = S.preset(name)
+    if T:
+        cfg = cfg.replace(T=T)
+    return cfg
+
+
+def describe(cfg) -> str:
+    act = "GELU" if cfg.act == 0 else "SwiGLU"
+    s = (f"{cfg.name}: T={cfg.T} d={cfg.d} E={cfg.E} {act} d_ff={cfg.d_ff} top-{cfg.k} K={cfg.n_groups} "
+         f"allowed={cfg.n_allowed}/{cfg.E} r={cfg.r}")
+    if cfg.n_shared:
+        s += f" shared={cfg.n_shared}x{cfg.d_ff_shared}"
+    return s
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ------------------------------------------------------------------ algorithmic work per launch
+def kernel_work(cfg, name: str):
+    """(flops, bytes) of one launch of a named kernel, from the layer shape.
+
+    GEMM bytes count the weights of the allowed experts once plus activations
+    read and written once; gate bytes count X, the gate weights and the Top-k
+    outputs; data-movement kernels count each row read and written once.
+    """
+    es = 2 if cfg.dtype == 1 else 4
+    T, d, k, E, r, ff = cfg.T, cfg.d, cfg.k, cfg.E, cfg.r, cfg.d_ff
+    n = T * k
+    na = cfg.n_allowed
+    glu = 2 if cfg.act == 1 else 1
+    K = cfg.n_groups if cfg.n_groups > 1 else 0
+    if name == "expert_up":
+        return 2.0 * n * d * ff * glu, es * (na * glu * ff * d + n * d + n * ff)
+    if name == "expert_down":
+        return 2.0 * n * ff * d, es * (na * d * ff + n * ff + n * d)
+    fs = cfg.d_ff_shared
+    if name == "shared_up":
+        return 2.0 * T * cfg.n_shared * d * fs * glu, es * (cfg.n_shared * glu * fs * d + T * d + T * cfg.n_shared * fs)
+    if name == "shared_down":
+        return 2.0 * T * cfg.n_shared * fs * d, es * (cfg.n_shared * d * fs + T * cfg.n_shared * (fs + d))
+    if name == "lr_encode":
+        return 2.0 * T * d * r, es * (T * d + r * d + T * r)
+    if name == "lr_decode":
+        return 2.0 * T * r * d, es * (T * r + d * r + T * d)
+    if name == "gate_topk":
+        return 2.0 * T * d * (E + K), es * T * d + 4 * (E + K) * d + 8 * n
+    if name == "gather_rows":
+        return 0.0, 2 * es * n * d + 4 * n
+    if name == "combine":
+        return 0.0, es * (n * d + cfg.n_shared * T * d + T * d)
+    if name in ("route_count", "route_scatter"):
+        return 0.0, 4 * n * (1 if name == "route_count" else 3)
+    return 0.0, 0.0
+
+
+def roofline_for(cfg, name, avg_ms, peaks, peaks_src, traffic):
+    flops, byts = kernel_work(cfg, name)
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    tensor = name in ("expert_up", "expert_down", "shared_up", "shared_down") or (
+        name in ("lr_encode", "lr_decode") and flops / max(byts, 1) >= ridge)
+    sec = avg_ms * 1e-3
+    if tensor and cfg.dtype == 1:
+        achieved = flops / sec / 1e12
+        peak = peaks["bf16_tflops"]
+        return {"kernel": name, "bound": "tensor", "achieved": round(achieved, 2), "peak": peak,
+                "unit": "TFLOP/s", "frac": round(achieved / peak, 4), "traffic": traffic,
+                "peak_source": f"{peaks_src} bf16 burst", "algorithmic_flops": flops, "avg_ms": round(avg_ms, 5)}
+    achieved = byts / sec / 1e9
+    peak = peaks["hbm_gbs"]
+    return {"kernel": name, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+            "frac": round(achieved / peak, 4), "traffic": traffic, "peak_source": f"{peaks_src} HBM copy",
+            "algorithmic_bytes": byts, "avg_ms": round(avg_ms, 5)}
+
+
+def committed_traffic(cfg, kernel):
+    """dram read+write bytes per launch for (workload, kernel) from profiles/traffic.txt, or None."""
+    p = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) >= 3 and not line.startswith("#") and parts[0] == cfg.name and parts[1] == kernel:
+                return float(parts[2])
+    return None
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi samples of the GPU's SM clock and throttle reasons during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str):
+        self.uuid = uuid
+        self.rows = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.uuid, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.rows.append([c.strip() for c in line.split(",")])
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=5)
+        sm, mx = [], []
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in self.rows:
+            try:
+                sm.append(float(r[0]))
+                mx.append(float(r[1]))
+            except (ValueError, IndexError):
+                continue
+            for nm, v in zip(names, r[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ reference arm (fp64 oracle on CPU)
+def oracle_sample_step(cfg, o, rows):
+    from oracle import ec2moe_oracle as orc
+    sub = dict(o)
+    sub["X"] = o["X"][rows]
+    return orc.layer_forward(sub, cfg.n_groups, cfg.k, cfg.act, bool(cfg.renorm_topk))
+
+
+def oracle_inputs_cpu(cfg):
+    from paper_2508_06024_gb300 import synth as S
+    inp = S.make_inputs(cfg, device="cpu")
+    out = {}
+    for k, v in inp.items():
+        if v is None:
+            out[k] = None
+        elif k == "mask":
+            out[k] = v.numpy().astype("uint8")
+        else:
+            out[k] = S.to_f64(v)
+    return out
+
+
+def time_oracle(cfg, budget_s: float, steps: int = 0):
+    """Tokens/s of the oracle on a bounded sample of the workload's tokens.
+
+    Returns (tokens_per_s, sample_desc, per_step_seconds list)."""
+    import numpy as np
+    o = oracle_inputs_cpu(cfg)
+    rng = np.random.default_rng(0)
+    # size the sample from a small probe so one step takes about budget_s / max(steps, 1)
+    probe = np.sort(rng.choice(cfg.T, min(64, cfg.T), replace=False))
+    t0 = time.perf_counter()
+    oracle_sample_step(cfg, o, probe)
+    per_tok = (time.perf_counter() - t0) / len(probe)
+    n_steps = max(steps, 1)
+    target = budget_s / n_steps
+    n_tok = int(min(cfg.T, max(16, target / max(per_tok, 1e-9))))
+    times = []
+    done = 0
+    for i in range(n_steps):
+        rows = np.sort(rng.choice(cfg.T, n_tok, replace=False))
+        t0 = time.perf_counter()
+        oracle_sample_step(cfg, o, rows)
+        times.append(time.perf_counter() - t0)
+        done += n_tok
+    total = sum(times)
+    desc = (f"{n_steps} x {n_tok} of {cfg.T} tokens (seeded sample; full layer on those tokens: gate, Top-k, "
+            f"routing tables, codec, experts, combine), numpy float64")
+    return done / total, desc, times, n_tok
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    cfg = workload_config(args.workload, args.T)
+    cores = os.cpu_count()
+    budget = max(10.0, min(120.0, 3.0 * (args.steps + args.warmup)))
+    tps, desc, times, n_tok = time_oracle(cfg, budget, steps=args.steps)
+    ms = 1e3 * cfg.T / tps
+    line = {"impl": "reference", "metric": METRIC, "value": round(tps, 2), "unit": "tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": describe(cfg), "l2": "n/a (CPU)"},
+            "cpu_baseline": {"value": round(tps, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": round(tps, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ our arm
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2508_06024_gb300 import build as B
+    from paper_2508_06024_gb300 import ec2moe as C
+    from paper_2508_06024_gb300 import synth as S
+    from paper_2508_06024_gb300.runner import LayerRun
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if rank == 0:
+        B.build()
+    if world > 1:
+        dist.barrier()
+    C.load()
+
+    cfg = workload_config(args.workload, args.T).replace(seed=rank)
+    inp = S.make_inputs(cfg, device=dev)
+    run = LayerRun(cfg, inp, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    for _ in range(max(args.warmup, 3)):
+        run.forward(stream=stream)
+    status = C.ec2moe_last_device_error(stream)
+    if status != C.OK:
+        raise RuntimeError(f"device error after warm-up: {C.status_string(status)}")
+    launches_per_step = C.ec2moe_last_launch_count()
+
+    def timed_loop(step_fn):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        barrier()
+        for i in range(args.steps):
+            flush.zero_()
+            evs[i][0].record(stream)
+            step_fn()
+            evs[i][1].record(stream)
+        barrier()
+        return [a.elapsed_time(b) for a, b in evs]
+
+    clocks = None
+    sampler = None
+    if rank == 0:
+        try:
+            uuid = str(torch.cuda.get_device_properties(dev).uuid)
+            uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+            sampler = ClockSampler(uuid)
+            sampler.start()
+            time.sleep(0.3)
+        except Exception:
+            sampler = None
+    step_ms = timed_loop(lambda: run.forward(stream=stream))
+    if sampler:
+        clocks = sampler.stop()
+    status = C.ec2moe_last_device_error(stream)
+    if status != C.OK:
+        raise RuntimeError(f"device error in the timed loop: {C.status_string(status)}")
+
+    # End to end through the public call: pinned host X -> device, layer, Y -> pinned host.
+    X_host = inp["X"].to("cpu").pin_memory()
+    Y_host = torch.empty(run.Y.shape, dtype=run.Y.dtype).pin_memory()
+    X_dev = torch.empty_like(inp["X"])
+
+    def e2e_step():
+        X_dev.copy_(X_host, non_blocking=True)
+        run.forward(X=X_dev, stream=stream)
+        Y_host.copy_(run.Y, non_blocking=True)
+
+    for _ in range(3):
+        e2e_step()
+    e2e_ms = timed_loop(e2e_step)
+
+    # Per-kernel device time: the same steps with every launch bracketed by events.
+    C.ec2moe_profile_reset()
+    C.ec2moe_profile_enable(True)
+    prof_steps = max(args.steps, 5)
+    barrier()
+    for _ in range(prof_steps):
+        flush.zero_()
+        run.forward(stream=stream)
+    barrier()
+    C.ec2moe_profile_enable(False)
+    per_kernel = {}
+    for i in range(C.ec2moe_profile_count()):
+        name, ms = C.ec2moe_profile_read(i)
+        per_kernel.setdefault(name, []).append(ms)
+    C.ec2moe_profile_reset()
+
+    total_ms = torch.tensor([sum(step_ms), sum(e2e_ms)], dtype=torch.float64, device=dev)
+    if world > 1:
+        dist.all_reduce(total_ms, op=dist.ReduceOp.MAX)
+    t_step = total_ms[0].item() / args.steps
+    t_e2e = total_ms[1].item() / args.steps
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return 0
+
+    peaks, peaks_src = load_peaks()
+    kern = {n: {"launches_per_step": len(v) / prof_steps, "avg_ms": statistics.mean(v),
+                "share": 0.0} for n, v in per_kernel.items()}
+    tot = sum(k["avg_ms"] * k["launches_per_step"] for k in kern.values())
+    for k in kern.values():
+        k["share"] = round(k["avg_ms"] * k["launches_per_step"] / tot, 4) if tot else 0.0
+        k["avg_ms"] = round(k["avg_ms"], 5)
+    dominant = max(kern, key=lambda n: kern[n]["avg_ms"] * kern[n]["launches_per_step"])
+    roof = roofline_for(cfg, dominant, kern[dominant]["avg_ms"], peaks, peaks_src,
+                        committed_traffic(cfg, dominant))
+    others = {n: roofline_for(cfg, n, kern[n]["avg_ms"], peaks, peaks_src, committed_traffic(cfg, n))
+              for n in kern}
+    layer_flops = sum(kernel_work(cfg, n)[0] * kern[n]["launches_per_step"] for n in kern)
+
+    cpu = None
+    if not args.no_cpu_baseline and world == 1:
+        tps, desc, _, _ = time_oracle(cfg, args.cpu_seconds, steps=1)
+        cpu = {"value": round(tps, 2), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": desc}
+
+    value = world * cfg.T / (t_step * 1e-3)
+    es = 2 if cfg.dtype == 1 else 4
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(t_step, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if cfg.dtype == 1 else "f32", "data": "synthetic",
+        "config": {"workload": describe(cfg), "l2": "flushed between steps (256 MiB write)",
+                   "parallelism": f"token-parallel replicas x{world}"},
+        "layer_tflops": round(layer_flops / (t_step * 1e-3) / 1e12, 2),
+        "layer_frac_bf16_peak": round(layer_flops / (t_step * 1e-3) / 1e12 / peaks["bf16_tflops"], 4),
+        "roofline": roof,
+        "kernels": {n: dict(kern[n], bound=others[n]["bound"], achieved=others[n]["achieved"],
+                            unit=others[n]["unit"], frac=others[n]["frac"]) for n in sorted(kern)},
+        "cpu_baseline": cpu,
+        "e2e": {"value": round(world * cfg.T / (t_e2e * 1e-3), 1), "unit": "tokens/s",
+                "h2d_bytes_per_step": cfg.T * cfg.d * es, "d2h_bytes_per_step": cfg.T * cfg.d * es,
+                "ms_per_step": round(t_e2e, 5)},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+        "peaks": {"source": peaks_src, "hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"]},
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

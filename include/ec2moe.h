@@ -1,0 +1,233 @@
+/*
+ * ec2moe.h - C ABI of libec2moe.so, the GB300 (sm_103a) MoE-layer forward of
+ * EC^2MoE (arXiv 2508.06024).
+ *
+ * The layer computes Eq. 1, y = sum_i G(x)_i E_i(x), with the gate G of the
+ * hardware-aware lightweight group gate network (Eq. 4 local candidate set,
+ * Eq. 5 per-group softmax gates, Eq. 6 global group gate, Eq. 7 fusion), Top-k
+ * routing (Top-1 in the paper's evaluation), and the low-rank encoder/decoder
+ * of the end-cloud pipeline (Z = U^T X V at the end, X_hat = U_hat Z V_hat^T in
+ * the cloud) at the split between gate/routing and the experts.
+ *
+ * Conventions shared by every entry point:
+ *  - Device pointers are CUDA device addresses owned by the caller; the library
+ *    never allocates, frees or keeps them.  Host pointers are marked "host".
+ *  - Matrices are row-major and dense.  Weights are stored [out, in], i.e. the
+ *    reduction axis is contiguous.  Every device pointer handed to a bf16
+ *    tensor-core GEMM must be 16-byte aligned and every row a multiple of 16
+ *    bytes (d, d_ff, r multiples of 8 for bf16); violations return
+ *    EC2MOE_ERR_MISALIGNED before any launch.
+ *  - Storage type: desc->dtype selects bf16 (EC2MOE_BF16) or fp32 (EC2MOE_F32)
+ *    for activations, expert weights and codec weights.  Gate weights and
+ *    biases are always fp32.  bf16 GEMMs accumulate in fp32.
+ *  - All work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *    stream).  No call synchronises except ec2moe_last_device_error.
+ *  - Arguments are validated on the host before any launch; a failed check
+ *    returns its status and enqueues nothing.  Kernels never trap: waits inside
+ *    the tensor-core kernels are bounded and report through a device error
+ *    word that ec2moe_last_device_error reads.
+ *  - Calls are thread-safe with respect to each other as long as they do not
+ *    share output buffers.
+ */
+#ifndef EC2MOE_H
+#define EC2MOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* ec2moe_stream_t; /* == cudaStream_t */
+
+typedef enum ec2moe_status {
+  EC2MOE_OK = 0,
+  EC2MOE_ERR_INVALID_ARG = 1,      /* NULL pointer, non-positive size, E % n_groups != 0, ... */
+  EC2MOE_ERR_ALL_MASKED = 2,       /* the local candidate set of Eq. 4 is empty */
+  EC2MOE_ERR_TOO_FEW_EXPERTS = 3,  /* k > number of allowed experts */
+  EC2MOE_ERR_UNSUPPORTED = 4,      /* a size beyond the limits below */
+  EC2MOE_ERR_CUDA = 5,             /* a CUDA runtime call failed */
+  EC2MOE_ERR_TIMEOUT = 6,          /* a bounded device wait gave up (see ec2moe_last_device_error) */
+  EC2MOE_ERR_WORKSPACE = 7,        /* workspace NULL or smaller than ec2moe_workspace_size */
+  EC2MOE_ERR_MISALIGNED = 8        /* pointer or row pitch not 16-byte aligned */
+} ec2moe_status;
+
+typedef enum ec2moe_dtype { EC2MOE_F32 = 0, EC2MOE_BF16 = 1 } ec2moe_dtype;
+
+/* Expert FFN activation: GELU(u) = u Phi(u) (exact erf form), or SwiGLU
+ * h = SiLU(W1 x) * (W3 x). */
+typedef enum ec2moe_act { EC2MOE_GELU = 0, EC2MOE_SWIGLU = 1 } ec2moe_act;
+
+#define EC2MOE_MAX_EXPERTS 128  /* E */
+#define EC2MOE_MAX_GROUPS 16    /* K, n_groups */
+#define EC2MOE_MAX_TOPK 8       /* k */
+#define EC2MOE_MAX_SHARED 4     /* n_shared */
+
+/* Shape of one MoE layer call.
+ *  T            tokens (rows of X), >= 0 (T = 0 is a no-op)
+ *  d            d_model
+ *  E            routed experts (M of Eq. 5)
+ *  d_ff         hidden width of each routed expert
+ *  k            experts per token (Top-k)
+ *  n_groups     K of Eq. 5-7; experts form K contiguous groups of E/K (group j
+ *               owns experts [j*E/K, (j+1)*E/K)).  K = 1 is the plain softmax gate.
+ *  act          ec2moe_act
+ *  dtype        ec2moe_dtype
+ *  r            codec rank; 0 = no codec (experts see X itself)
+ *  n_shared     always-on shared experts (weight 1, not masked, not counted)
+ *  d_ff_shared  hidden width of each shared expert
+ *  renorm_topk  0: the combine weight is g_i itself (Eq. 1 with G = g);
+ *               1: g_i divided by the sum of g over the token's top-k */
+typedef struct ec2moe_layer_desc {
+  int32_t T, d, E, d_ff, k, n_groups;
+  int32_t act, dtype;
+  int32_t r;
+  int32_t n_shared, d_ff_shared;
+  int32_t renorm_topk;
+} ec2moe_layer_desc;
+
+/* Weights of one layer (device pointers, NULL where absent).
+ *  W_local  fp32 [E, d]  the group gates W_k of Eq. 5 stacked in group order
+ *  b_local  fp32 [E]     the b_k of Eq. 5 stacked likewise
+ *  W_global fp32 [K, d]  Eq. 6 (NULL iff K == 1)
+ *  b_global fp32 [K]     Eq. 6 (NULL iff K == 1)
+ *  W1, W3   [E, d_ff, d] up projections (W3 only for SwiGLU)
+ *  W2       [E, d, d_ff] down projection
+ *  W1s, W3s [n_shared, d_ff_shared, d]; W2s [n_shared, d, d_ff_shared]
+ *  V_enc    [r, d]       encoder: Z = X V_enc^T (V of the codec, U = I on tokens)
+ *  V_dec    [d, r]       decoder: X_hat = Z V_dec^T (V_hat, U_hat = I) */
+typedef struct ec2moe_layer_weights {
+  const float* W_local;
+  const float* b_local;
+  const float* W_global;
+  const float* b_global;
+  const void* W1;
+  const void* W3;
+  const void* W2;
+  const void* W1s;
+  const void* W3s;
+  const void* W2s;
+  const void* V_enc;
+  const void* V_dec;
+} ec2moe_layer_weights;
+
+/* Bytes of device workspace ec2moe_layer_forward needs for `desc` (0 on an
+ * invalid desc).  The workspace holds the codec output Z, the decoded and
+ * expert-ordered activations, the expert hidden activations, per-slot expert
+ * outputs and the routing tables. */
+size_t ec2moe_workspace_size(const ec2moe_layer_desc* desc);
+
+/* Bytes of device workspace ec2moe_experts needs (hidden activations). */
+size_t ec2moe_experts_workspace_size(const ec2moe_layer_desc* desc);
+
+/* Bytes of device workspace ec2moe_route needs (per-block histograms). */
+size_t ec2moe_route_workspace_size(const ec2moe_layer_desc* desc);
+
+/* Steps 1-3a: local expert filter, group gate and Top-k (Eq. 4-7).
+ *  X         [T, d] activations (dtype)
+ *  mask      host uint8 [E]; 1 = expert in the local candidate set of Eq. 4.
+ *            An all-zero mask returns EC2MOE_ERR_ALL_MASKED and fewer than k
+ *            ones EC2MOE_ERR_TOO_FEW_EXPERTS.
+ *  topk_idx  out int32 [T, k] expert ids, slot 0 = largest g, ties to the
+ *            lower expert index
+ *  topk_w    out fp32 [T, k] combine weights (g_i, or renormalised over the
+ *            top-k when desc->renorm_topk)
+ * Within a group the order is decided on the fp32 local logits; across groups
+ * on the fp32 fused log-probability log p_group + log p_local. */
+ec2moe_status ec2moe_gate(const ec2moe_layer_desc* desc, const void* X, const float* W_local,
+                          const float* b_local, const float* W_global, const float* b_global,
+                          const uint8_t* mask, int32_t* topk_idx, float* topk_w,
+                          ec2moe_stream_t stream);
+
+/* Step 3b: per-expert histogram, exclusive scan and stable permutation, plus
+ * the optional gather of activation rows into expert order.
+ *  topk_idx  int32 [T, k] (from ec2moe_gate)
+ *  counts    out int32 [E]     tokens routed to each expert
+ *  offsets   out int32 [E + 1] exclusive prefix sum of counts
+ *  perm      out int32 [T * k] perm[p] = t * k + s for the p-th row in
+ *            expert-major order; rows of one expert keep increasing (t, s)
+ *  inv_perm  out int32 [T * k] or NULL: inv_perm[perm[p]] = p
+ *  src, dst  NULL, or src [T, width] and dst [T * k, width] (dtype):
+ *            dst[p] = src[perm[p] / k]
+ *  workspace device scratch of ec2moe_route_workspace_size bytes */
+ec2moe_status ec2moe_route(const ec2moe_layer_desc* desc, const int32_t* topk_idx, int32_t* counts,
+                           int32_t* offsets, int32_t* perm, int32_t* inv_perm, const void* src,
+                           int32_t width, void* dst, void* workspace, size_t ws_bytes,
+                           ec2moe_stream_t stream);
+
+/* Steps 4-5a: routed expert FFNs on expert-ordered rows with the gate scale and
+ * the unpermute fused into the down projection.
+ *  X_perm    [T * k, d] rows in expert order (ec2moe_route's dst)
+ *  offsets   int32 [E + 1] device (ec2moe_route)
+ *  perm      int32 [T * k] device (ec2moe_route)
+ *  topk_w    fp32 [T, k] (ec2moe_gate)
+ *  slot_out  out [T * k, d]: slot_out[t * k + s] = topk_w[t, s] * E_e(x_t)
+ *            for e = topk_idx[t, s]
+ *  workspace ec2moe_experts_workspace_size bytes */
+ec2moe_status ec2moe_experts(const ec2moe_layer_desc* desc, const void* X_perm, const int32_t* offsets,
+                             const void* W1, const void* W3, const void* W2, const float* topk_w,
+                             const int32_t* perm, void* slot_out, void* workspace, size_t ws_bytes,
+                             ec2moe_stream_t stream);
+
+/* Always-on shared experts on every token: shared_out[s * T + t] = E_s(x_t).
+ *  X [T, d]; W1s/W3s/W2s as in ec2moe_layer_weights; shared_out out
+ *  [n_shared * T, d]; workspace of ec2moe_experts_workspace_size bytes. */
+ec2moe_status ec2moe_shared_experts(const ec2moe_layer_desc* desc, const void* X, const void* W1s,
+                                    const void* W3s, const void* W2s, void* shared_out, void* workspace,
+                                    size_t ws_bytes, ec2moe_stream_t stream);
+
+/* Step 5b: y[t] = sum_s slot_out[t * k + s] + sum_j shared_out[j * T + t], in
+ * that fixed order with an fp32 sum (Eq. 1).  shared_out may be NULL. */
+ec2moe_status ec2moe_combine(const ec2moe_layer_desc* desc, const void* slot_out, const void* shared_out,
+                             void* Y, ec2moe_stream_t stream);
+
+/* Step 6, end side: Z = X V_enc^T ([T, d] x [r, d]^T -> [T, r]). */
+ec2moe_status ec2moe_lr_encode(const ec2moe_layer_desc* desc, const void* X, const void* V_enc, void* Z,
+                               ec2moe_stream_t stream);
+
+/* Step 6, cloud side: X_hat = Z V_dec^T ([T, r] x [d, r]^T -> [T, d]). */
+ec2moe_status ec2moe_lr_decode(const ec2moe_layer_desc* desc, const void* Z, const void* V_dec,
+                               void* X_hat, ec2moe_stream_t stream);
+
+/* The fused layer: gate and routing on X, encode, decode into expert order,
+ * routed and shared experts, combine.
+ *  Y         out [T, d] (dtype)
+ *  topk_idx  out int32 [T, k]; topk_w out fp32 [T, k]; counts out int32 [E]
+ *  Z         out [T, r] or NULL: the transmitted (encoded) activations
+ *  workspace ec2moe_workspace_size(desc) bytes */
+ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_layer_weights* w,
+                                   const void* X, const uint8_t* mask, void* Y, int32_t* topk_idx,
+                                   float* topk_w, int32_t* counts, void* Z, void* workspace,
+                                   size_t ws_bytes, ec2moe_stream_t stream);
+
+/* Synchronises `stream`, then reads and clears the device error word of the
+ * current device: EC2MOE_OK, EC2MOE_ERR_TIMEOUT when a bounded wait in a
+ * tensor-core kernel gave up, or EC2MOE_ERR_CUDA when the stream reports an
+ * error. */
+ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream);
+
+/* Number of kernels the last successful call on this host thread enqueued. */
+int32_t ec2moe_last_launch_count(void);
+
+/* Per-launch timing.  While enabled, every kernel the library enqueues is
+ * bracketed by a pair of CUDA events recorded on its stream; records
+ * accumulate until ec2moe_profile_reset.  Reading a record synchronises on its
+ * stop event.  `name` receives a static string naming the launch
+ * ("gate_topk", "route_count", "route_scatter", "gather_rows", "lr_encode",
+ * "lr_decode", "expert_up", "expert_down", "shared_up", "shared_down",
+ * "combine"); `ms` its device duration.  Profiling is off by default and
+ * costs nothing when off. */
+ec2moe_status ec2moe_profile_enable(int32_t enable);
+int32_t ec2moe_profile_count(void);
+ec2moe_status ec2moe_profile_read(int32_t i, const char** name, float* ms);
+void ec2moe_profile_reset(void);
+
+/* Human-readable name of a status code (static storage). */
+const char* ec2moe_status_string(ec2moe_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EC2MOE_H */

@@ -1,0 +1,589 @@
+// C ABI of libec2moe.so (declared in include/ec2moe.h): host-side argument
+// checks, workspace layout and the order of launches for each step of the
+// EC^2MoE MoE-layer forward.
+#include <cuda_runtime.h>
+
+#include <mutex>
+#include <vector>
+
+#include "../../include/ec2moe.h"
+#include "internal.h"
+
+namespace ec2moe {
+
+namespace {
+thread_local int t_launches = 0;
+
+// Per-launch timing records (ec2moe_profile_*).  Events come from a pool that
+// is reused after ec2moe_profile_reset.
+struct ProfRecord {
+  const char* name;
+  cudaEvent_t start, stop;
+};
+std::mutex g_prof_mu;
+bool g_prof_on = false;
+std::vector<ProfRecord> g_prof;
+std::vector<cudaEvent_t> g_pool;
+size_t g_pool_used = 0;
+
+cudaEvent_t pool_event() {
+  if (g_pool_used == g_pool.size()) {
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    g_pool.push_back(e);
+  }
+  return g_pool[g_pool_used++];
+}
+}  // namespace
+
+void reset_launch_count() { t_launches = 0; }
+int launch_count() { return t_launches; }
+
+KernelScope::KernelScope(const char* name, cudaStream_t s) : name_(name), s_(s) {
+  std::lock_guard<std::mutex> lock(g_prof_mu);
+  if (g_prof_on) {
+    start_ = pool_event();
+    if (start_) cudaEventRecord(start_, s_);
+  }
+}
+
+KernelScope::~KernelScope() {
+  ++t_launches;
+  std::lock_guard<std::mutex> lock(g_prof_mu);
+  if (g_prof_on && start_) {
+    cudaEvent_t stop = pool_event();
+    if (stop) {
+      cudaEventRecord(stop, s_);
+      g_prof.push_back(ProfRecord{name_, start_, stop});
+    }
+  }
+}
+
+int sm_count() {
+  static std::mutex mu;
+  static std::vector<int> cache;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  std::lock_guard<std::mutex> lock(mu);
+  if ((int)cache.size() <= dev) cache.resize(dev + 1, 0);
+  if (cache[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+    cache[dev] = n;
+  }
+  return cache[dev];
+}
+
+}  // namespace ec2moe
+
+using namespace ec2moe;
+
+namespace {
+
+constexpr size_t ALIGN = 256;
+size_t align_up(size_t x) { return (x + ALIGN - 1) / ALIGN * ALIGN; }
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t esize(const ec2moe_layer_desc* d) { return d->dtype == EC2MOE_BF16 ? 2 : 4; }
+bool is_bf16(const ec2moe_layer_desc* d) { return d->dtype == EC2MOE_BF16; }
+
+// Shape checks common to every entry point.
+ec2moe_status check_desc(const ec2moe_layer_desc* d) {
+  if (!d) return EC2MOE_ERR_INVALID_ARG;
+  if (d->T < 0 || d->d <= 0 || d->E <= 0 || d->k <= 0 || d->n_groups <= 0 || d->r < 0 || d->n_shared < 0)
+    return EC2MOE_ERR_INVALID_ARG;
+  if (d->dtype != EC2MOE_F32 && d->dtype != EC2MOE_BF16) return EC2MOE_ERR_INVALID_ARG;
+  if (d->act != EC2MOE_GELU && d->act != EC2MOE_SWIGLU) return EC2MOE_ERR_INVALID_ARG;
+  if (d->renorm_topk != 0 && d->renorm_topk != 1) return EC2MOE_ERR_INVALID_ARG;
+  if (d->E % d->n_groups != 0) return EC2MOE_ERR_INVALID_ARG;
+  if (d->k > d->E) return EC2MOE_ERR_TOO_FEW_EXPERTS;
+  if (d->E > EC2MOE_MAX_EXPERTS || d->n_groups > EC2MOE_MAX_GROUPS || d->k > EC2MOE_MAX_TOPK ||
+      d->n_shared > EC2MOE_MAX_SHARED)
+    return EC2MOE_ERR_UNSUPPORTED;
+  if ((long long)d->T * d->k + (long long)d->T * (d->n_shared + 1) > 0x7fffffffLL) return EC2MOE_ERR_UNSUPPORTED;
+  // Row pitches must be multiples of 16 bytes (vector loads, TMA strides) and,
+  // for the tensor-core path, output widths multiples of 32 columns.
+  if (d->d % 8 != 0) return EC2MOE_ERR_MISALIGNED;
+  return EC2MOE_OK;
+}
+
+ec2moe_status check_ffn(const ec2moe_layer_desc* d, int d_ff) {
+  if (d_ff <= 0) return EC2MOE_ERR_INVALID_ARG;
+  if (d_ff % 8 != 0) return EC2MOE_ERR_MISALIGNED;
+  if (is_bf16(d) && (d_ff % 32 != 0 || d->d % 32 != 0)) return EC2MOE_ERR_UNSUPPORTED;
+  return EC2MOE_OK;
+}
+
+ec2moe_status check_codec(const ec2moe_layer_desc* d) {
+  if (d->r <= 0) return EC2MOE_ERR_INVALID_ARG;
+  if (d->r % 8 != 0) return EC2MOE_ERR_MISALIGNED;
+  if (is_bf16(d) && (d->r % 32 != 0 || d->d % 32 != 0)) return EC2MOE_ERR_UNSUPPORTED;
+  return EC2MOE_OK;
+}
+
+ec2moe_status check_mask(const ec2moe_layer_desc* d, const uint8_t* mask, uint32_t bits[4]) {
+  if (!mask) return EC2MOE_ERR_INVALID_ARG;
+  bits[0] = bits[1] = bits[2] = bits[3] = 0;
+  int n = 0;
+  for (int e = 0; e < d->E; ++e)
+    if (mask[e]) {
+      bits[e >> 5] |= 1u << (e & 31);
+      ++n;
+    }
+  if (n == 0) return EC2MOE_ERR_ALL_MASKED;
+  if (n < d->k) return EC2MOE_ERR_TOO_FEW_EXPERTS;
+  return EC2MOE_OK;
+}
+
+#define EC2MOE_REQUIRE_PTR(p)                   \
+  do {                                          \
+    if (!(p)) return EC2MOE_ERR_INVALID_ARG;    \
+    if (!aligned16(p)) return EC2MOE_ERR_MISALIGNED; \
+  } while (0)
+
+#define EC2MOE_CUDA(call)                        \
+  do {                                           \
+    if ((call) != cudaSuccess) return EC2MOE_ERR_CUDA; \
+  } while (0)
+
+// Workspace of ec2moe_layer_forward, each region 256-byte aligned.
+struct LayerWs {
+  size_t z, xa, h, slot, shared, perm, inv_perm, offsets, blk, total;
+};
+LayerWs layer_ws(const ec2moe_layer_desc* d) {
+  LayerWs w{};
+  const size_t es = esize(d);
+  const size_t T = d->T, k = d->k, dm = d->d;
+  const size_t ff = d->d_ff > d->d_ff_shared ? d->d_ff : d->d_ff_shared;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t at = off;
+    off += align_up(bytes);
+    return at;
+  };
+  w.z = take(d->r > 0 ? T * d->r * es : 0);
+  w.xa = take((T * k + T) * dm * es);                          // expert-ordered rows, then X_hat
+  w.h = take((T * k + (size_t)d->n_shared * T) * ff * es);    // hidden activations
+  const bool direct = (d->k == 1 && d->n_shared == 0);
+  w.slot = take(direct ? 0 : T * k * dm * es);
+  w.shared = take((size_t)d->n_shared * T * dm * es);
+  w.perm = take(T * k * 4);
+  w.inv_perm = take(T * k * 4);
+  w.offsets = take((d->E + 1) * 4);
+  w.blk = take((size_t)route_blocks((long long)T * k) * d->E * 4);
+  w.total = off;
+  return w;
+}
+
+GemmArgs gemm_base() {
+  GemmArgs g{};
+  g.timeout_cycles = default_timeout_cycles();
+  return g;
+}
+
+cudaError_t run_gemm(const ec2moe_layer_desc* d, const GemmArgs& g, int epi, cudaStream_t s) {
+  return is_bf16(d) ? launch_gemm_tc(g, epi, s) : launch_gemm_simt(g, epi, s);
+}
+
+// Up projection (+ activation) then down projection over groups of rows.
+//   routed: groups = experts by device offsets; down projection scatters with
+//           perm and scales with the gate weights.
+//   shared: groups = shared experts, each over all T rows of A.
+cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long long a_rows, long long a_row_base,
+                    const int32_t* offsets, const void* W1, const void* W3, const void* W2, void* H, long long h_rows,
+                    long long h_row_base, const int32_t* perm, const float* scale, void* out, long long out_row_base,
+                    cudaStream_t s) {
+  const int ff = routed ? d->d_ff : d->d_ff_shared;
+  const int G = routed ? d->E : d->n_shared;
+  const long long rows = routed ? (long long)d->T * d->k : (long long)d->T * d->n_shared;
+  const int act_epi = d->act == EC2MOE_SWIGLU ? EPI_SWIGLU : EPI_GELU;
+  GemmArgs up = gemm_base();
+  up.name = routed ? "expert_up" : "shared_up";
+  up.A = A;
+  up.a_rows = a_rows;
+  up.B = W1;
+  up.B2 = W3;
+  up.b_rows = (long long)G * ff;
+  up.offsets = routed ? offsets : nullptr;
+  up.G = G;
+  up.M = routed ? 0 : d->T;
+  up.a_shared = routed ? 0 : 1;
+  up.a_row_base = a_row_base;
+  up.out_row_base = h_row_base;
+  up.N = ff;
+  up.K = d->d;
+  up.b_group_rows = ff;
+  up.out = H;
+  up.ldo = ff;
+  up.max_rows = rows;
+  cudaError_t e = run_gemm(d, up, act_epi, s);
+  if (e != cudaSuccess) return e;
+  GemmArgs dn = gemm_base();
+  dn.name = routed ? "expert_down" : "shared_down";
+  dn.A = H;
+  dn.a_rows = h_rows;
+  dn.B = W2;
+  dn.B2 = nullptr;
+  dn.b_rows = (long long)G * d->d;
+  dn.offsets = routed ? offsets : nullptr;
+  dn.G = G;
+  dn.M = routed ? 0 : d->T;
+  dn.a_shared = 0;
+  dn.a_row_base = h_row_base;
+  dn.out_row_base = routed ? 0 : out_row_base;
+  dn.N = d->d;
+  dn.K = ff;
+  dn.b_group_rows = d->d;
+  dn.out = out;
+  dn.ldo = d->d;
+  dn.perm = routed ? perm : nullptr;
+  dn.scale = routed ? scale : nullptr;
+  dn.max_rows = rows;
+  return run_gemm(d, dn, routed ? EPI_SCATTER : EPI_STORE, s);
+}
+
+cudaError_t run_codec(const ec2moe_layer_desc* d, bool encode, const void* in, const void* V, void* out,
+                      cudaStream_t s) {
+  GemmArgs g = gemm_base();
+  g.name = encode ? "lr_encode" : "lr_decode";
+  g.A = in;
+  g.a_rows = d->T;
+  g.B = V;
+  g.b_rows = encode ? d->r : d->d;
+  g.G = 1;
+  g.M = d->T;
+  g.N = encode ? d->r : d->d;
+  g.K = encode ? d->d : d->r;
+  g.b_group_rows = 0;
+  g.out = out;
+  g.ldo = g.N;
+  g.max_rows = d->T;
+  return run_gemm(d, g, EPI_STORE, s);
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t ec2moe_workspace_size(const ec2moe_layer_desc* desc) {
+  if (check_desc(desc) != EC2MOE_OK) return 0;
+  return layer_ws(desc).total;
+}
+
+size_t ec2moe_experts_workspace_size(const ec2moe_layer_desc* desc) {
+  if (check_desc(desc) != EC2MOE_OK) return 0;
+  const size_t T = desc->T, k = desc->k;
+  const size_t routed = T * k * desc->d_ff;
+  const size_t shared = (size_t)desc->n_shared * T * desc->d_ff_shared;
+  return align_up((routed > shared ? routed : shared) * esize(desc));
+}
+
+size_t ec2moe_route_workspace_size(const ec2moe_layer_desc* desc) {
+  if (check_desc(desc) != EC2MOE_OK) return 0;
+  return align_up((size_t)route_blocks((long long)desc->T * desc->k) * desc->E * 4);
+}
+
+ec2moe_status ec2moe_gate(const ec2moe_layer_desc* desc, const void* X, const float* W_local, const float* b_local,
+                          const float* W_global, const float* b_global, const uint8_t* mask, int32_t* topk_idx,
+                          float* topk_w, ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  GateArgs a{};
+  st = check_mask(desc, mask, a.mask_bits);
+  if (st != EC2MOE_OK) return st;
+  if (desc->T == 0) return EC2MOE_OK;
+  EC2MOE_REQUIRE_PTR(X);
+  EC2MOE_REQUIRE_PTR(W_local);
+  EC2MOE_REQUIRE_PTR(b_local);
+  EC2MOE_REQUIRE_PTR(topk_idx);
+  EC2MOE_REQUIRE_PTR(topk_w);
+  if (desc->n_groups > 1) {
+    EC2MOE_REQUIRE_PTR(W_global);
+    EC2MOE_REQUIRE_PTR(b_global);
+  }
+  a.X = X;
+  a.W_local = W_local;
+  a.b_local = b_local;
+  a.W_global = desc->n_groups > 1 ? W_global : nullptr;
+  a.b_global = desc->n_groups > 1 ? b_global : nullptr;
+  a.T = desc->T;
+  a.d = desc->d;
+  a.E = desc->E;
+  a.K = desc->n_groups;
+  a.k = desc->k;
+  a.renorm = desc->renorm_topk;
+  a.topk_idx = topk_idx;
+  a.topk_w = topk_w;
+  EC2MOE_CUDA(launch_gate(a, is_bf16(desc), stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_route(const ec2moe_layer_desc* desc, const int32_t* topk_idx, int32_t* counts, int32_t* offsets,
+                           int32_t* perm, int32_t* inv_perm, const void* src, int32_t width, void* dst,
+                           void* workspace, size_t ws_bytes, ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  if (!counts || !offsets) return EC2MOE_ERR_INVALID_ARG;
+  if ((src == nullptr) != (dst == nullptr)) return EC2MOE_ERR_INVALID_ARG;
+  if (src) {
+    if (width <= 0) return EC2MOE_ERR_INVALID_ARG;
+    if ((width * esize(desc)) % 16 != 0 || !aligned16(src) || !aligned16(dst)) return EC2MOE_ERR_MISALIGNED;
+  }
+  const long long n = (long long)desc->T * desc->k;
+  if (n > 0) {
+    if (!topk_idx || !perm) return EC2MOE_ERR_INVALID_ARG;
+    if (!workspace || ws_bytes < ec2moe_route_workspace_size(desc)) return EC2MOE_ERR_WORKSPACE;
+  }
+  EC2MOE_CUDA(launch_route(topk_idx, n, desc->E, static_cast<int32_t*>(workspace), counts, offsets, perm, inv_perm,
+                           stream));
+  if (src && n > 0) EC2MOE_CUDA(launch_gather(src, dst, perm, n, desc->k, width, is_bf16(desc), stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_experts(const ec2moe_layer_desc* desc, const void* X_perm, const int32_t* offsets, const void* W1,
+                             const void* W3, const void* W2, const float* topk_w, const int32_t* perm, void* slot_out,
+                             void* workspace, size_t ws_bytes, ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  st = check_ffn(desc, desc->d_ff);
+  if (st != EC2MOE_OK) return st;
+  if (desc->T == 0) return EC2MOE_OK;
+  EC2MOE_REQUIRE_PTR(X_perm);
+  EC2MOE_REQUIRE_PTR(W1);
+  EC2MOE_REQUIRE_PTR(W2);
+  if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(W3);
+  EC2MOE_REQUIRE_PTR(slot_out);
+  if (!offsets || !topk_w || !perm) return EC2MOE_ERR_INVALID_ARG;
+  if (!workspace || ws_bytes < ec2moe_experts_workspace_size(desc)) return EC2MOE_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return EC2MOE_ERR_MISALIGNED;
+  const long long rows = (long long)desc->T * desc->k;
+  EC2MOE_CUDA(run_ffn(desc, true, X_perm, rows, 0, offsets, W1, W3, W2, workspace, rows, 0, perm, topk_w, slot_out, 0,
+                      stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_shared_experts(const ec2moe_layer_desc* desc, const void* X, const void* W1s, const void* W3s,
+                                    const void* W2s, void* shared_out, void* workspace, size_t ws_bytes,
+                                    ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  if (desc->n_shared == 0) return EC2MOE_OK;
+  st = check_ffn(desc, desc->d_ff_shared);
+  if (st != EC2MOE_OK) return st;
+  if (desc->T == 0) return EC2MOE_OK;
+  EC2MOE_REQUIRE_PTR(X);
+  EC2MOE_REQUIRE_PTR(W1s);
+  EC2MOE_REQUIRE_PTR(W2s);
+  if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(W3s);
+  EC2MOE_REQUIRE_PTR(shared_out);
+  if (!workspace || ws_bytes < ec2moe_experts_workspace_size(desc)) return EC2MOE_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return EC2MOE_ERR_MISALIGNED;
+  const long long hrows = (long long)desc->T * desc->n_shared;
+  EC2MOE_CUDA(run_ffn(desc, false, X, desc->T, 0, nullptr, W1s, W3s, W2s, workspace, hrows, 0, nullptr, nullptr,
+                      shared_out, 0, stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_combine(const ec2moe_layer_desc* desc, const void* slot_out, const void* shared_out, void* Y,
+                             ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  if (desc->T == 0) return EC2MOE_OK;
+  EC2MOE_REQUIRE_PTR(slot_out);
+  EC2MOE_REQUIRE_PTR(Y);
+  if (shared_out && !aligned16(shared_out)) return EC2MOE_ERR_MISALIGNED;
+  EC2MOE_CUDA(launch_combine(slot_out, shared_out, desc->n_shared, Y, desc->T, desc->k, desc->d, is_bf16(desc), stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_lr_encode(const ec2moe_layer_desc* desc, const void* X, const void* V_enc, void* Z,
+                               ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  st = check_codec(desc);
+  if (st != EC2MOE_OK) return st;
+  if (desc->T == 0) return EC2MOE_OK;
+  EC2MOE_REQUIRE_PTR(X);
+  EC2MOE_REQUIRE_PTR(V_enc);
+  EC2MOE_REQUIRE_PTR(Z);
+  EC2MOE_CUDA(run_codec(desc, true, X, V_enc, Z, stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_lr_decode(const ec2moe_layer_desc* desc, const void* Z, const void* V_dec, void* X_hat,
+                               ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  st = check_codec(desc);
+  if (st != EC2MOE_OK) return st;
+  if (desc->T == 0) return EC2MOE_OK;
+  EC2MOE_REQUIRE_PTR(Z);
+  EC2MOE_REQUIRE_PTR(V_dec);
+  EC2MOE_REQUIRE_PTR(X_hat);
+  EC2MOE_CUDA(run_codec(desc, false, Z, V_dec, X_hat, stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_layer_weights* w, const void* X,
+                                   const uint8_t* mask, void* Y, int32_t* topk_idx, float* topk_w, int32_t* counts,
+                                   void* Z, void* workspace, size_t ws_bytes, ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  if (!w) return EC2MOE_ERR_INVALID_ARG;
+  GateArgs ga{};
+  st = check_mask(desc, mask, ga.mask_bits);
+  if (st != EC2MOE_OK) return st;
+  st = check_ffn(desc, desc->d_ff);
+  if (st != EC2MOE_OK) return st;
+  if (desc->n_shared > 0) {
+    st = check_ffn(desc, desc->d_ff_shared);
+    if (st != EC2MOE_OK) return st;
+  }
+  if (desc->r > 0) {
+    st = check_codec(desc);
+    if (st != EC2MOE_OK) return st;
+  }
+  if (desc->T == 0) return EC2MOE_OK;
+  EC2MOE_REQUIRE_PTR(X);
+  EC2MOE_REQUIRE_PTR(Y);
+  EC2MOE_REQUIRE_PTR(topk_idx);
+  EC2MOE_REQUIRE_PTR(topk_w);
+  if (!counts) return EC2MOE_ERR_INVALID_ARG;
+  EC2MOE_REQUIRE_PTR(w->W_local);
+  EC2MOE_REQUIRE_PTR(w->b_local);
+  if (desc->n_groups > 1) {
+    EC2MOE_REQUIRE_PTR(w->W_global);
+    EC2MOE_REQUIRE_PTR(w->b_global);
+  }
+  EC2MOE_REQUIRE_PTR(w->W1);
+  EC2MOE_REQUIRE_PTR(w->W2);
+  if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(w->W3);
+  if (desc->n_shared > 0) {
+    EC2MOE_REQUIRE_PTR(w->W1s);
+    EC2MOE_REQUIRE_PTR(w->W2s);
+    if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(w->W3s);
+  }
+  if (desc->r > 0) {
+    EC2MOE_REQUIRE_PTR(w->V_enc);
+    EC2MOE_REQUIRE_PTR(w->V_dec);
+    if (Z && !aligned16(Z)) return EC2MOE_ERR_MISALIGNED;
+  }
+  const LayerWs L = layer_ws(desc);
+  if (!workspace || ws_bytes < L.total) return EC2MOE_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return EC2MOE_ERR_MISALIGNED;
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  const bool bf = is_bf16(desc);
+  const size_t es = esize(desc);
+  const long long T = desc->T, k = desc->k, n = T * k;
+  void* zbuf = (desc->r > 0) ? (Z ? Z : ws + L.z) : nullptr;
+  uint8_t* xa = ws + L.xa;                      // [n + T, d]
+  uint8_t* x_hat = xa + (size_t)n * desc->d * es;  // rows [n, n + T)
+  void* h = ws + L.h;
+  const bool direct = (k == 1 && desc->n_shared == 0);
+  void* slot = direct ? Y : static_cast<void*>(ws + L.slot);
+  void* shared = desc->n_shared > 0 ? static_cast<void*>(ws + L.shared) : nullptr;
+  int32_t* perm = reinterpret_cast<int32_t*>(ws + L.perm);
+  int32_t* inv_perm = reinterpret_cast<int32_t*>(ws + L.inv_perm);
+  int32_t* offsets = reinterpret_cast<int32_t*>(ws + L.offsets);
+  int32_t* blk = reinterpret_cast<int32_t*>(ws + L.blk);
+
+  // Steps 1-3a on the end: mask, group gate, Top-k on the original activations.
+  ga.X = X;
+  ga.W_local = w->W_local;
+  ga.b_local = w->b_local;
+  ga.W_global = desc->n_groups > 1 ? w->W_global : nullptr;
+  ga.b_global = desc->n_groups > 1 ? w->b_global : nullptr;
+  ga.T = desc->T;
+  ga.d = desc->d;
+  ga.E = desc->E;
+  ga.K = desc->n_groups;
+  ga.k = desc->k;
+  ga.renorm = desc->renorm_topk;
+  ga.topk_idx = topk_idx;
+  ga.topk_w = topk_w;
+  EC2MOE_CUDA(launch_gate(ga, bf, stream));
+  // Step 3b: routing tables.
+  EC2MOE_CUDA(launch_route(topk_idx, n, desc->E, blk, counts, offsets, perm, inv_perm, stream));
+  // Step 6: encode at the end, decode in the cloud (experts read X_hat).
+  if (desc->r > 0) {
+    EC2MOE_CUDA(run_codec(desc, true, X, w->V_enc, zbuf, stream));
+    EC2MOE_CUDA(run_codec(desc, false, zbuf, w->V_dec, x_hat, stream));
+  } else {
+    EC2MOE_CUDA(cudaMemcpyAsync(x_hat, X, (size_t)T * desc->d * es, cudaMemcpyDeviceToDevice, stream));
+  }
+  // Step 3b (move): rows into expert order.
+  EC2MOE_CUDA(launch_gather(x_hat, xa, perm, n, desc->k, desc->d, bf, stream));
+  // Steps 4-5a: routed experts, gate scale and unpermute fused in the down projection.
+  EC2MOE_CUDA(run_ffn(desc, true, xa, n + T, 0, offsets, w->W1, w->W3, w->W2, h, n + (long long)desc->n_shared * T, 0,
+                      perm, topk_w, slot, 0, stream));
+  // Always-on shared experts on X_hat.
+  if (desc->n_shared > 0) {
+    EC2MOE_CUDA(run_ffn(desc, false, xa, n + T, n, nullptr, w->W1s, w->W3s, w->W2s, h,
+                        n + (long long)desc->n_shared * T, n, nullptr, nullptr, shared, 0, stream));
+  }
+  // Step 5b: fixed-order combine (skipped when the down projection wrote Y directly).
+  if (!direct) EC2MOE_CUDA(launch_combine(slot, shared, desc->n_shared, Y, desc->T, desc->k, desc->d, bf, stream));
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream) {
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  unsigned int word = 0;
+  if (read_tc_error(&word) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  return word ? EC2MOE_ERR_TIMEOUT : EC2MOE_OK;
+}
+
+int32_t ec2moe_last_launch_count(void) { return launch_count(); }
+
+ec2moe_status ec2moe_profile_enable(int32_t enable) {
+  std::lock_guard<std::mutex> lock(g_prof_mu);
+  g_prof_on = enable != 0;
+  return EC2MOE_OK;
+}
+
+int32_t ec2moe_profile_count(void) {
+  std::lock_guard<std::mutex> lock(g_prof_mu);
+  return static_cast<int32_t>(g_prof.size());
+}
+
+ec2moe_status ec2moe_profile_read(int32_t i, const char** name, float* ms) {
+  std::lock_guard<std::mutex> lock(g_prof_mu);
+  if (i < 0 || i >= (int32_t)g_prof.size() || !name || !ms) return EC2MOE_ERR_INVALID_ARG;
+  const ProfRecord& r = g_prof[i];
+  if (cudaEventSynchronize(r.stop) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (cudaEventElapsedTime(ms, r.start, r.stop) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  *name = r.name;
+  return EC2MOE_OK;
+}
+
+void ec2moe_profile_reset(void) {
+  std::lock_guard<std::mutex> lock(g_prof_mu);
+  g_prof.clear();
+  g_pool_used = 0;
+}
+
+const char* ec2moe_status_string(ec2moe_status s) {
+  switch (s) {
+    case EC2MOE_OK: return "ok";
+    case EC2MOE_ERR_INVALID_ARG: return "invalid argument";
+    case EC2MOE_ERR_ALL_MASKED: return "all experts masked";
+    case EC2MOE_ERR_TOO_FEW_EXPERTS: return "fewer allowed experts than k";
+    case EC2MOE_ERR_UNSUPPORTED: return "unsupported size";
+    case EC2MOE_ERR_CUDA: return "CUDA error";
+    case EC2MOE_ERR_TIMEOUT: return "device wait timed out";
+    case EC2MOE_ERR_WORKSPACE: return "workspace too small";
+    case EC2MOE_ERR_MISALIGNED: return "misaligned pointer or pitch";
+  }
+  return "unknown status";
+}
+
+}  // extern "C"

@@ -1,0 +1,86 @@
+// Internal launch interfaces shared by the translation units of libec2moe.so.
+// Nothing here is exported; the public ABI is include/ec2moe.h.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace ec2moe {
+
+// Kernels enqueued by the current public call on this host thread.
+void reset_launch_count();
+int launch_count();
+
+// Wraps one kernel launch: counts it and, while profiling is enabled
+// (ec2moe_profile_enable), brackets it with CUDA events on its stream.
+class KernelScope {
+ public:
+  KernelScope(const char* name, cudaStream_t s);
+  ~KernelScope();
+  KernelScope(const KernelScope&) = delete;
+  KernelScope& operator=(const KernelScope&) = delete;
+
+ private:
+  const char* name_;
+  cudaStream_t s_;
+  cudaEvent_t start_ = nullptr;
+};
+
+int sm_count();
+
+// ----------------------------------------------------------------- gate (Eq. 4-7)
+struct GateArgs {
+  const void* X;  // [T, d] bf16 or fp32
+  const float* W_local;
+  const float* b_local;
+  const float* W_global;  // nullptr when K == 1
+  const float* b_global;
+  uint32_t mask_bits[4];  // bit e = expert e allowed (E <= 128)
+  int T, d, E, K, k, renorm;
+  int32_t* topk_idx;
+  float* topk_w;
+};
+cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s);
+
+// ----------------------------------------------------------- routing tables / moves
+int route_blocks(long long n_entries);  // per-block histogram blocks
+cudaError_t launch_route(const int32_t* topk_idx, long long n_entries, int E, int32_t* blk_counts,
+                         int32_t* counts, int32_t* offsets, int32_t* perm, int32_t* inv_perm,
+                         cudaStream_t s);
+// dst[p] = src[perm[p] / k] for p < rows, width elements per row.
+cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long long rows, int k, int width,
+                          bool bf16, cudaStream_t s);
+// y[t] = sum_s slot[t*k+s] + sum_j shared[j*T+t]
+cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d,
+                           bool bf16, cudaStream_t s);
+
+// ------------------------------------------------------------------ grouped GEMMs
+enum Epi { EPI_STORE = 0, EPI_GELU = 1, EPI_SWIGLU = 2, EPI_SCATTER = 3 };
+
+// Group g of a grouped GEMM owns rows [row0(g), row0(g) + M_g) of A and of the
+// pre-scatter output, with
+//   offsets != nullptr: row0 = offsets[g], M_g = offsets[g+1] - offsets[g]
+//   offsets == nullptr: M_g = M, row0_out = g*M, row0_A = a_shared ? 0 : g*M
+// both shifted by a_row_base / out_row_base.  Group g multiplies by rows
+// [g*b_group_rows, g*b_group_rows + N) of B (and of B2 for SwiGLU).
+struct GemmArgs {
+  const void* A; long long a_rows;   // A [a_rows, K]
+  const void* B; const void* B2; long long b_rows;  // B, B2 [b_rows, K]
+  const int32_t* offsets; int G; int M; int a_shared;
+  long long a_row_base, out_row_base;
+  int N, K, b_group_rows;
+  void* out; long long ldo;          // output pitch in elements
+  const int32_t* perm;               // EPI_SCATTER: dest row = perm[out_row]
+  const float* scale;                // EPI_SCATTER: multiply by scale[dest] (nullptr = 1)
+  long long max_rows;                // upper bound of sum_g M_g (for the grid size)
+  long long timeout_cycles;          // bounded-wait budget (tensor-core path)
+  const char* name;                  // label for per-launch profiling (nullptr = by epilogue)
+};
+cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s);    // bf16, tcgen05
+cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s);  // fp32, CUDA cores
+// Reads and clears the tensor-core kernels' device error word (synchronous).
+cudaError_t read_tc_error(unsigned int* word);
+long long default_timeout_cycles();
+
+}  // namespace ec2moe

@@ -1,0 +1,198 @@
+// Step 3b and step 5b of the layer: per-expert histogram, exclusive scan and
+// stable expert-major permutation of the (token, slot) pairs chosen by Top-k;
+// the row gather into expert order; and the fixed-order combine of Eq. 1.
+//
+// Routing runs as two kernels over blocks of CHUNK consecutive (token, slot)
+// entries:
+//   count    shared-memory atomic histogram per block -> blk_counts[b][e]
+//   scatter  each block derives its expert bases from the column sums of
+//            blk_counts, ranks its entries stably inside the block
+//            (warp match + popc, then a prefix over the block's warps) and
+//            writes perm / inv_perm; block 0 also writes counts and offsets.
+// Rows of one expert therefore keep increasing (t, s) order, which makes the
+// permutation (and everything downstream) deterministic.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace ec2moe {
+namespace {
+
+constexpr int CHUNK = 1024;  // entries per block (one per thread)
+constexpr int MAXE = 128;
+
+__global__ void __launch_bounds__(CHUNK) route_count_kernel(const int32_t* __restrict__ idx, long long n, int E,
+                                                            int32_t* __restrict__ blk_counts) {
+  __shared__ int hist[MAXE];
+  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[e] = 0;
+  __syncthreads();
+  const long long i = (long long)blockIdx.x * CHUNK + threadIdx.x;
+  if (i < n) atomicAdd(&hist[idx[i]], 1);
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x) blk_counts[(long long)blockIdx.x * E + e] = hist[e];
+}
+
+__global__ void __launch_bounds__(CHUNK) route_scatter_kernel(const int32_t* __restrict__ idx, long long n, int E,
+                                                              const int32_t* __restrict__ blk_counts, int nblk,
+                                                              int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
+                                                              int32_t* __restrict__ perm, int32_t* __restrict__ inv_perm) {
+  __shared__ int s_pre[MAXE];           // entries of expert e in earlier blocks
+  __shared__ int s_base[MAXE];          // offsets[e] + s_pre[e]
+  __shared__ int s_tot[MAXE];
+  __shared__ int s_wcnt[CHUNK / 32][MAXE];  // per-warp counts, then per-warp exclusive prefix
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  for (int i = threadIdx.x; i < (CHUNK / 32) * MAXE; i += blockDim.x) (&s_wcnt[0][0])[i] = 0;
+  for (int e = threadIdx.x; e < E; e += blockDim.x) {
+    int pre = 0, tot = 0;
+    for (int b = 0; b < nblk; ++b) {
+      const int c = blk_counts[(long long)b * E + e];
+      if (b < (int)blockIdx.x) pre += c;
+      tot += c;
+    }
+    s_pre[e] = pre;
+    s_tot[e] = tot;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int e = 0; e < E; ++e) {
+      const int c = s_tot[e];
+      s_base[e] = acc + s_pre[e];
+      if (blockIdx.x == 0) {
+        counts[e] = c;
+        offsets[e] = acc;
+      }
+      acc += c;
+    }
+    if (blockIdx.x == 0) offsets[E] = acc;
+  }
+  const long long i = (long long)blockIdx.x * CHUNK + threadIdx.x;
+  const bool live = i < n;
+  const unsigned act = __ballot_sync(0xffffffffu, live);
+  int e = -1, rank_w = 0;
+  if (live) {
+    e = idx[i];
+    const unsigned same = __match_any_sync(act, e);
+    rank_w = __popc(same & ((1u << lane) - 1u));
+    if (rank_w == 0) s_wcnt[warp][e] = __popc(same);
+  }
+  __syncthreads();
+  for (int ee = threadIdx.x; ee < E; ee += blockDim.x) {
+    int acc = 0;
+    for (int w = 0; w < CHUNK / 32; ++w) {
+      const int c = s_wcnt[w][ee];
+      s_wcnt[w][ee] = acc;
+      acc += c;
+    }
+  }
+  __syncthreads();
+  if (live) {
+    const int pos = s_base[e] + s_wcnt[warp][e] + rank_w;
+    perm[pos] = static_cast<int32_t>(i);
+    if (inv_perm) inv_perm[i] = pos;
+  }
+}
+
+// dst[p] = src[perm[p] / k]; one warp per row, 16-byte lanes.
+__global__ void gather_rows_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
+                                   const int32_t* __restrict__ perm, long long rows, int k, int row_bytes) {
+  const int lane = threadIdx.x & 31;
+  const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
+  for (long long r = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += warps) {
+    const long long t = perm[r] / k;
+    const U4* s = reinterpret_cast<const U4*>(src + t * row_bytes);
+    U4* d = reinterpret_cast<U4*>(dst + r * row_bytes);
+    for (int c = lane; c < row_bytes / 16; c += 32) d[c] = s[c];
+  }
+}
+
+// y[t] = sum_s slot[t*k+s] + sum_j shared[j*T+t] in that order, fp32 sum.
+template <typename TE>
+__global__ void combine_kernel(const TE* __restrict__ slot, const TE* __restrict__ shared, int n_shared,
+                               TE* __restrict__ Y, int T, int k, int d) {
+  const int per_row = d / 8;
+  const long long total = (long long)T * per_row;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (long long)gridDim.x * blockDim.x) {
+    const long long t = i / per_row;
+    const int c = static_cast<int>(i % per_row) * 8;
+    float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+    float v[8];
+    for (int s = 0; s < k; ++s) {
+      load8(slot + (t * k + s) * d + c, v);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] += v[j];
+    }
+    for (int j = 0; j < n_shared; ++j) {
+      load8(shared + ((long long)j * T + t) * d + c, v);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] += v[q];
+    }
+    store8(Y + t * d + c, acc);
+  }
+}
+
+}  // namespace
+
+int route_blocks(long long n_entries) { return static_cast<int>((n_entries + CHUNK - 1) / CHUNK); }
+
+cudaError_t launch_route(const int32_t* topk_idx, long long n, int E, int32_t* blk_counts, int32_t* counts,
+                         int32_t* offsets, int32_t* perm, int32_t* inv_perm, cudaStream_t s) {
+  const int nblk = route_blocks(n);
+  if (nblk == 0) {
+    // No entries: counts = 0, offsets = 0.
+    cudaError_t e = cudaMemsetAsync(counts, 0, sizeof(int32_t) * E, s);
+    if (e != cudaSuccess) return e;
+    return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
+  }
+  {
+    KernelScope ks("route_count", s);
+    route_count_kernel<<<nblk, CHUNK, 0, s>>>(topk_idx, n, E, blk_counts);
+  }
+  {
+    KernelScope ks("route_scatter", s);
+    route_scatter_kernel<<<nblk, CHUNK, 0, s>>>(topk_idx, n, E, blk_counts, nblk, counts, offsets, perm, inv_perm);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long long rows, int k, int width, bool bf16,
+                          cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  const int row_bytes = width * (bf16 ? 2 : 4);
+  const int warps_per_block = 8;
+  long long blocks = (rows + warps_per_block - 1) / warps_per_block;
+  const long long cap = (long long)sm_count() * 8;
+  if (blocks > cap) blocks = cap;
+  {
+    KernelScope ks("gather_rows", s);
+    gather_rows_kernel<<<static_cast<int>(blocks), warps_per_block * 32, 0, s>>>(
+        static_cast<const uint8_t*>(src), static_cast<uint8_t*>(dst), perm, rows, k, row_bytes);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d, bool bf16,
+                           cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  const long long total = (long long)T * (d / 8);
+  long long blocks = (total + 255) / 256;
+  const long long cap = (long long)sm_count() * 8;
+  if (blocks > cap) blocks = cap;
+  KernelScope ks("combine", s);
+  if (bf16) {
+    combine_kernel<__nv_bfloat16><<<static_cast<int>(blocks), 256, 0, s>>>(
+        static_cast<const __nv_bfloat16*>(slot), static_cast<const __nv_bfloat16*>(shared), shared ? n_shared : 0,
+        static_cast<__nv_bfloat16*>(Y), T, k, d);
+  } else {
+    combine_kernel<float><<<static_cast<int>(blocks), 256, 0, s>>>(static_cast<const float*>(slot),
+                                                                   static_cast<const float*>(shared),
+                                                                   shared ? n_shared : 0, static_cast<float*>(Y), T, k, d);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace ec2moe

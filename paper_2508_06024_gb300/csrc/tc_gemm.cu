@@ -1,0 +1,530 @@
+// Grouped bf16 GEMM on the sm_103a tensor cores: tcgen05.mma with the fp32
+// accumulator in tensor memory (TMEM), operands staged by TMA into 128-byte
+// swizzled shared memory, and a persistent warp-specialised CTA per SM.
+//
+// Used for the expert FFN projections (Eq. 1 experts, steps 4-5) and the
+// low-rank codec projections (Z = X V_enc^T, X_hat = Z V_dec^T).  Every group g
+// computes  C_g = A_g B_g^T  with A_g [M_g, K] (rows of A) and B_g [N, K]
+// (rows of a weight matrix stored [out, in]), and the epilogue applies the
+// step-specific op (plain store, GELU, SwiGLU, or gate-scale + scatter to the
+// token's slot for the combine of Eq. 1).
+//
+// CTA layout (192 threads):
+//   warp 0      TMA producer (one elected lane)
+//   warp 1      TMEM allocator + MMA issuer (one elected lane)
+//   warps 2..5  epilogue: TMEM -> registers -> global (warp w reads TMEM lanes
+//               32*(w%4) .. +31, i.e. rows of the 128-row tile)
+// Pipelines: STAGES shared-memory stages (full/empty mbarriers) and two TMEM
+// accumulators (tmem_full/tmem_empty) so the epilogue of tile i overlaps the
+// main loop of tile i+1.
+//
+// Every mbarrier wait is bounded by a clock64 budget.  A wait that gives up
+// sets the device error word, raises a CTA-wide abort flag that ends every
+// other wait at once, waits (again bounded) for the CTA's own TMA copies and
+// MMAs still in flight, frees TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <mutex>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace ec2moe {
+
+__device__ unsigned int g_tc_error;  // bit 0: a bounded wait timed out
+
+namespace {
+
+constexpr int BM = 128;   // tile rows (MMA M, TMEM lanes)
+constexpr int BK = 64;    // K per stage: one 128-byte swizzle row of bf16
+constexpr int UK = 16;    // K of one tcgen05.mma kind::f16
+constexpr int NUM_THREADS = 192;
+constexpr int MAX_GROUPS = 136;
+
+struct Params {
+  const int32_t* offsets;
+  int G, M, a_shared;
+  long long a_row_base, out_row_base;
+  int N, K, b_group_rows;
+  void* out;
+  long long ldo;
+  const int32_t* perm;
+  const float* scale;
+  long long timeout;
+  int n_tiles_n;
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}\n"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait.  Returns false when the budget ran out or another role of the
+// CTA already aborted (it then also raises the abort flag and the error word).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long long budget, volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (clock64() - t0 > budget) {
+      *abort_flag = 1;
+      atomicOr(&g_tc_error, 1u);
+      return false;
+    }
+  }
+}
+// Wait used while draining after an abort: bounded, ignores the abort flag.
+__device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity, long long budget) {
+  const long long t0 = clock64();
+  while (!mbar_try_wait(bar, parity)) {
+    if (clock64() - t0 > budget) return;
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor (tcgen05 format) for a K-major operand tile
+// stored as rows of 128 bytes with the 128-byte swizzle, 8-row atoms 1024 bytes
+// apart.  Fields: start address >> 4 (bits 0-13), leading byte offset >> 4
+// (16-29, unused for swizzled K-major), stride byte offset >> 4 (32-45),
+// descriptor version 1 (46-47), base offset 0 (49-51), swizzle mode 2 =
+// 128-byte (61-63).
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(1) << 16;
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;
+  d |= static_cast<uint64_t>(1) << 46;
+  d |= static_cast<uint64_t>(2) << 61;
+  return d;
+}
+// Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator (bits 4-5
+// = 1), A and B bf16 (bits 7-9 and 10-12 = 1), both K-major (bits 15, 16 = 0),
+// N >> 3 in bits 17-22, M >> 4 in bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(m >> 4) << 24);
+}
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t da, uint64_t db, uint32_t idesc, uint32_t accum) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(da), "l"(db), "r"(idesc), "r"(accum)
+      : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+// 32 lanes x 32 columns of 32-bit TMEM words: thread i of the warp receives
+// columns [col, col+32) of TMEM lane (quadrant base + i).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// ------------------------------------------------------------------ tile schedule
+struct TileCoord {
+  int g, m_blk, n_blk;
+};
+
+// Linear tile order: group-major, then n block, then m block, so CTAs that run
+// at the same time share the group's weight tiles and activation rows in L2.
+__device__ __forceinline__ TileCoord decode_tile(int tile, const int* tile_prefix, int n_tiles_n, int& cursor) {
+  while (tile >= tile_prefix[cursor + 1] * n_tiles_n) ++cursor;
+  const int mt = tile_prefix[cursor + 1] - tile_prefix[cursor];
+  const int rem = tile - tile_prefix[cursor] * n_tiles_n;
+  return TileCoord{cursor, rem % mt, rem / mt};
+}
+
+template <int BN, int EPI, int STAGES>
+struct Cfg {
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int BN_OUT = (EPI == EPI_SWIGLU) ? BN / 2 : BN;
+  static constexpr int TMEM_COLS = 2 * BN;  // two accumulators
+  static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8;
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES + 16 + 2 * (MAX_GROUPS + 1) * 4;
+};
+
+template <int BN, int EPI, int STAGES>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmB2, const Params p) {
+  using C = Cfg<BN, EPI, STAGES>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * C::A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + STAGES;
+  uint64_t* tfull = bars + 2 * STAGES;
+  uint64_t* tempty = bars + 2 * STAGES + 2;
+  uint64_t* drain = bars + 2 * STAGES + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 5);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* tile_prefix = reinterpret_cast<int*>(tmem_slot + 4);
+  int* row0 = tile_prefix + (MAX_GROUPS + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(smem_u32(&tfull[a]), 1);
+      mbar_init(smem_u32(&tempty[a]), 4);
+    }
+    mbar_init(smem_u32(drain), 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // Per-group tile prefix (m tiles) and first rows.
+    int acc = 0;
+    tile_prefix[0] = 0;
+    for (int g = 0; g < p.G; ++g) {
+      int r0, mg;
+      if (p.offsets) {
+        r0 = p.offsets[g];
+        mg = p.offsets[g + 1] - r0;
+      } else {
+        r0 = g * p.M;
+        mg = p.M;
+      }
+      row0[g] = r0;
+      acc += (mg + BM - 1) / BM;
+      tile_prefix[g + 1] = acc;
+    }
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+    if (EPI == EPI_SWIGLU) tma_prefetch_desc(&tmB2);
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(C::TMEM_COLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int n_tiles = tile_prefix[p.G] * p.n_tiles_n;
+  const int num_kb = (p.K + BK - 1) / BK;
+  const long long budget = p.timeout;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0;  // bit s: stage s holds a copy the consumer has not released
+      uint32_t issued_phase = 0;
+      int cursor = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+        const TileCoord tc = decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
+        const int a_row = static_cast<int>(p.a_row_base) + (p.offsets ? row0[tc.g] : (p.a_shared ? 0 : row0[tc.g])) +
+                          tc.m_blk * BM;
+        const int b_row = tc.g * p.b_group_rows + tc.n_blk * C::BN_OUT;
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1u, budget, abort_flag)) {
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_u32(&full[stage]);
+          mbar_expect_tx(fb, C::STAGE_BYTES);
+          tma_load_2d(smem_u32(sA + stage * C::A_BYTES), &tmA, kb * BK, a_row, fb);
+          if (EPI == EPI_SWIGLU) {
+            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK, b_row, fb);
+            tma_load_2d(smem_u32(sB + stage * C::B_BYTES + C::B_BYTES / 2), &tmB2, kb * BK, b_row, fb);
+          } else {
+            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK, b_row, fb);
+          }
+          issued |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      if (!ok || *abort_flag) {
+        // Let every copy this CTA started land before shared memory is released.
+        for (int s = 0; s < STAGES; ++s)
+          if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, budget);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t IDESC = idesc_bf16(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int it = 0;
+      int cursor = 0;
+      bool ok = true, any = false;
+      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++it) {
+        (void)decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
+        const int acc = it & 1;
+        const uint32_t acc_phase = (it >> 1) & 1;
+        if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, budget, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+        for (int kb = 0; kb < num_kb; ++kb) {
+          if (!mbar_wait(smem_u32(&full[stage]), phase, budget, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * C::B_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < BK / UK; ++kk) {
+            umma_bf16(d_tmem, sdesc_sw128(a0 + kk * UK * 2), sdesc_sw128(b0 + kk * UK * 2), IDESC,
+                      (kb | kk) != 0 ? 1u : 0u);
+          }
+          any = true;
+          umma_commit(smem_u32(&empty[stage]));
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(smem_u32(&tfull[acc]));
+      }
+      if ((!ok || *abort_flag) && any) {
+        // All MMAs issued so far must finish before TMEM is freed.
+        umma_commit(smem_u32(drain));
+        mbar_drain(smem_u32(drain), 0, budget);
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int row_in_tile = q * 32 + lane;
+    int it = 0;
+    int cursor = 0;
+    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++it) {
+      const TileCoord tc = decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
+      const int acc = it & 1;
+      const uint32_t acc_phase = (it >> 1) & 1;
+      if (!mbar_wait(smem_u32(&tfull[acc]), acc_phase, budget, abort_flag)) break;
+      tc_fence_after();
+      const int mg = p.offsets ? (p.offsets[tc.g + 1] - p.offsets[tc.g]) : p.M;
+      const int local = tc.m_blk * BM + row_in_tile;
+      const bool valid = local < mg;
+      const long long out_row = p.out_row_base + row0[tc.g] + local;
+      long long dest = out_row;
+      float sc = 1.0f;
+      if (EPI == EPI_SCATTER && valid) {
+        dest = p.perm ? p.perm[out_row] : out_row;
+        if (p.scale) sc = p.scale[dest];
+      }
+      const uint32_t t_row = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
+      __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out) + dest * p.ldo;
+#pragma unroll 1
+      for (int c0 = 0; c0 < C::BN_OUT; c0 += 32) {
+        const int col = tc.n_blk * C::BN_OUT + c0;
+        float v[32];
+        tmem_ld32(t_row + c0, v);
+        if (EPI == EPI_SWIGLU) {
+          float u[32];
+          tmem_ld32(t_row + c0 + BN / 2, u);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = silu(v[i]) * u[i];
+        } else if (EPI == EPI_GELU) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
+        } else if (EPI == EPI_SCATTER) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] *= sc;
+        }
+        if (valid && col < p.N) {
+#pragma unroll
+          for (int j = 0; j < 4; ++j) store8(orow + col + 8 * j, v + 8 * j);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(C::TMEM_COLS)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------------------------ host side
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix, box = 64 columns x box_rows
+// rows, 128-byte swizzle, zero fill out of bounds.
+bool make_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+const char* kernel_name(int epi) {
+  switch (epi) {
+    case EPI_GELU: return "gemm_tc_gelu";
+    case EPI_SWIGLU: return "gemm_tc_swiglu";
+    case EPI_SCATTER: return "gemm_tc_scatter";
+    default: return "gemm_tc_store";
+  }
+}
+
+template <int BN, int EPI, int STAGES>
+cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
+  using C = Cfg<BN, EPI, STAGES>;
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(tc_gemm_kernel<BN, EPI, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    C::SMEM);
+  });
+  if (attr_err != cudaSuccess) return attr_err;
+  CUtensorMap mA, mB, mB2;
+  const int b_box = (EPI == EPI_SWIGLU) ? BN / 2 : BN;
+  if (!make_map(&mA, a.A, a.a_rows, a.K, BM)) return cudaErrorInvalidValue;
+  if (!make_map(&mB, a.B, a.b_rows, a.K, b_box)) return cudaErrorInvalidValue;
+  if (EPI == EPI_SWIGLU) {
+    if (!make_map(&mB2, a.B2, a.b_rows, a.K, b_box)) return cudaErrorInvalidValue;
+  } else {
+    mB2 = mB;
+  }
+  Params p;
+  p.offsets = a.offsets;
+  p.G = a.G;
+  p.M = a.M;
+  p.a_shared = a.a_shared;
+  p.a_row_base = a.a_row_base;
+  p.out_row_base = a.out_row_base;
+  p.N = a.N;
+  p.K = a.K;
+  p.b_group_rows = a.b_group_rows;
+  p.out = a.out;
+  p.ldo = a.ldo;
+  p.perm = a.perm;
+  p.scale = a.scale;
+  p.timeout = a.timeout_cycles;
+  p.n_tiles_n = (a.N + C::BN_OUT - 1) / C::BN_OUT;
+  const long long m_tiles_max = a.max_rows / BM + a.G;
+  long long tiles = m_tiles_max * p.n_tiles_n;
+  int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
+  if (grid < 1) grid = 1;
+  KernelScope ks(a.name ? a.name : kernel_name(EPI), s);
+  tc_gemm_kernel<BN, EPI, STAGES><<<grid, NUM_THREADS, C::SMEM, s>>>(mA, mB, mB2, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
+  if (a.G < 1 || a.G > MAX_GROUPS || a.N % 32 != 0 || a.K % 8 != 0) return cudaErrorInvalidValue;
+  // Wide N tiles where N allows it; 128 otherwise.
+  const bool wide = (epi == EPI_SWIGLU) ? (a.N % 128 == 0) : (a.N % 256 == 0);
+  switch (epi) {
+    case EPI_STORE:
+      return wide ? launch_cfg<256, EPI_STORE, 4>(a, s) : launch_cfg<128, EPI_STORE, 6>(a, s);
+    case EPI_GELU:
+      return wide ? launch_cfg<256, EPI_GELU, 4>(a, s) : launch_cfg<128, EPI_GELU, 6>(a, s);
+    case EPI_SWIGLU:
+      return wide ? launch_cfg<256, EPI_SWIGLU, 4>(a, s) : launch_cfg<128, EPI_SWIGLU, 6>(a, s);
+    case EPI_SCATTER:
+      return wide ? launch_cfg<256, EPI_SCATTER, 4>(a, s) : launch_cfg<128, EPI_SCATTER, 6>(a, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t read_tc_error(unsigned int* word) {
+  unsigned int zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(word, g_tc_error, sizeof(unsigned int));
+  if (e != cudaSuccess) return e;
+  return cudaMemcpyToSymbol(g_tc_error, &zero, sizeof(unsigned int));
+}
+
+// About two seconds at the GB300's maximum SM clock.
+long long default_timeout_cycles() { return 4000000000LL; }
+
+}  // namespace ec2moe
