@@ -156,6 +156,34 @@ ec2moe_status ec2moe_route(const ec2moe_layer_desc* desc, const int32_t* topk_id
                            int32_t width, void* dst, void* workspace, size_t ws_bytes,
                            ec2moe_stream_t stream);
 
+/* ec2moe_route without a workspace argument, for callers that cannot allocate
+ * device memory: programs whose device memory is planned and reserved in full
+ * before they start (a serving process that hands every byte to its own pool),
+ * code in a latency-critical loop that must not hit cudaMalloc's implicit
+ * device synchronisation, and bindings from languages that have no device
+ * allocator of their own.  The paper has no counterpart; this is a library
+ * convenience.
+ *
+ * Same arguments, results and errors as ec2moe_route except `workspace` and
+ * `ws_bytes`.  The routing histograms live in a fixed 64 KiB device array
+ * inside the library (EC2MOE_ROUTE_NOALLOC_MAX_CELLS int32 cells, one per
+ * block of 1024 (token, slot) entries and expert), which every GPU that loads
+ * the library holds until the process exits.  Sizes with
+ * ceil(T * k / 1024) * E > EC2MOE_ROUTE_NOALLOC_MAX_CELLS (for E = 64: T * k >
+ * 262144) return EC2MOE_ERR_UNSUPPORTED before any launch.  Nothing is
+ * allocated or freed, by this call or by anything it calls.
+ *
+ * The first call on each device looks up the array's device address (with
+ * that device current) and caches it; make that first call before any stream
+ * capture.  All calls on a device share the array: every cell a call reads is
+ * written earlier by the same call, but calls whose kernels overlap on the GPU
+ * (different streams, or different host threads) race on it and must be
+ * serialised by the caller. */
+#define EC2MOE_ROUTE_NOALLOC_MAX_CELLS 16384
+ec2moe_status ec2moe_route_noalloc(const ec2moe_layer_desc* desc, const int32_t* topk_idx, int32_t* counts,
+                                   int32_t* offsets, int32_t* perm, int32_t* inv_perm, const void* src,
+                                   int32_t width, void* dst, ec2moe_stream_t stream);
+
 /* Steps 4-5a: routed expert FFNs on expert-ordered rows with the gate scale and
  * the unpermute fused into the down projection.
  *  X_perm    [T * k, d] rows in expert order (ec2moe_route's dst)

@@ -342,6 +342,26 @@ ec2moe_status ec2moe_route(const ec2moe_layer_desc* desc, const int32_t* topk_id
   return EC2MOE_OK;
 }
 
+ec2moe_status ec2moe_route_noalloc(const ec2moe_layer_desc* desc, const int32_t* topk_idx, int32_t* counts,
+                                   int32_t* offsets, int32_t* perm, int32_t* inv_perm, const void* src, int32_t width,
+                                   void* dst, ec2moe_stream_t stream) {
+  reset_launch_count();
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  if (!counts || !offsets) return EC2MOE_ERR_INVALID_ARG;
+  if ((src == nullptr) != (dst == nullptr)) return EC2MOE_ERR_INVALID_ARG;
+  if (src) {
+    if (width <= 0) return EC2MOE_ERR_INVALID_ARG;
+    if ((width * esize(desc)) % 16 != 0 || !aligned16(src) || !aligned16(dst)) return EC2MOE_ERR_MISALIGNED;
+  }
+  const long long n = (long long)desc->T * desc->k;
+  if ((long long)route_blocks(n) * desc->E > EC2MOE_ROUTE_NOALLOC_MAX_CELLS) return EC2MOE_ERR_UNSUPPORTED;
+  if (n > 0 && (!topk_idx || !perm)) return EC2MOE_ERR_INVALID_ARG;
+  EC2MOE_CUDA(launch_route_noalloc(topk_idx, n, desc->E, counts, offsets, perm, inv_perm, stream));
+  if (src && n > 0) EC2MOE_CUDA(launch_gather(src, dst, perm, n, desc->k, width, is_bf16(desc), stream));
+  return EC2MOE_OK;
+}
+
 ec2moe_status ec2moe_experts(const ec2moe_layer_desc* desc, const void* X_perm, const int32_t* offsets, const void* W1,
                              const void* W3, const void* W2, const float* topk_w, const int32_t* perm, void* slot_out,
                              void* workspace, size_t ws_bytes, ec2moe_stream_t stream) {

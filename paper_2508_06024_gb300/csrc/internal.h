@@ -48,6 +48,12 @@ int route_blocks(long long n_entries);  // per-block histogram blocks
 cudaError_t launch_route(const int32_t* topk_idx, long long n_entries, int E, int32_t* blk_counts,
                          int32_t* counts, int32_t* offsets, int32_t* perm, int32_t* inv_perm,
                          cudaStream_t s);
+// Same as launch_route, but the per-block histograms live in a fixed device
+// array inside the library instead of caller memory (ec2moe_route_noalloc).
+// Returns cudaErrorInvalidValue when ceil(n_entries / 1024) * E exceeds
+// EC2MOE_ROUTE_NOALLOC_MAX_CELLS.
+cudaError_t launch_route_noalloc(const int32_t* topk_idx, long long n_entries, int E, int32_t* counts,
+                                 int32_t* offsets, int32_t* perm, int32_t* inv_perm, cudaStream_t s);
 // dst[p] = src[perm[p] / k] for p < rows, width elements per row.
 cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long long rows, int k, int width,
                           bool bf16, cudaStream_t s);

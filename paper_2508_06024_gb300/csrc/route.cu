@@ -14,11 +14,22 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <mutex>
+
+#include "../../include/ec2moe.h"
 #include "common.cuh"
 #include "internal.h"
 
 namespace ec2moe {
 namespace {
+
+// Histogram cells of ec2moe_route_noalloc: one int32 per (block of 1024
+// entries, expert), EC2MOE_ROUTE_NOALLOC_MAX_CELLS of them (64 KiB).  Every GPU
+// that loads the library keeps this array until the process exits.  All calls
+// on a device share it; the count kernel writes every cell the scatter kernel
+// later reads, so nothing in it has to start at zero, but two calls whose
+// kernels overlap on the GPU race on it.
+static __device__ __align__(256) int32_t g_route_noalloc_cells[EC2MOE_ROUTE_NOALLOC_MAX_CELLS];
 
 constexpr int CHUNK = 1024;  // entries per block (one per thread)
 constexpr int MAXE = 128;
@@ -157,6 +168,37 @@ cudaError_t launch_route(const int32_t* topk_idx, long long n, int E, int32_t* b
     route_scatter_kernel<<<nblk, CHUNK, 0, s>>>(topk_idx, n, E, blk_counts, nblk, counts, offsets, perm, inv_perm);
   }
   return cudaGetLastError();
+}
+
+// Device address of g_route_noalloc_cells for the current device.  The host-side
+// name of a __device__ array is only a stand-in, so the address is looked up
+// once per device (with that device current) and cached.
+static cudaError_t noalloc_cells(int32_t** out) {
+  constexpr int MAX_DEVICES = 64;
+  static std::mutex mu;
+  static int32_t* cache[MAX_DEVICES] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= MAX_DEVICES) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!cache[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_route_noalloc_cells);
+    if (e != cudaSuccess) return e;
+    cache[dev] = static_cast<int32_t*>(p);
+  }
+  *out = cache[dev];
+  return cudaSuccess;
+}
+
+cudaError_t launch_route_noalloc(const int32_t* topk_idx, long long n, int E, int32_t* counts, int32_t* offsets,
+                                 int32_t* perm, int32_t* inv_perm, cudaStream_t s) {
+  if ((long long)route_blocks(n) * E > EC2MOE_ROUTE_NOALLOC_MAX_CELLS) return cudaErrorInvalidValue;
+  int32_t* cells = nullptr;
+  cudaError_t e = noalloc_cells(&cells);
+  if (e != cudaSuccess) return e;
+  return launch_route(topk_idx, n, E, cells, counts, offsets, perm, inv_perm, s);
 }
 
 cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long long rows, int k, int width, bool bf16,

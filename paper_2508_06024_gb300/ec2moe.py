@@ -39,7 +39,7 @@ EXPORTED = [
     "ec2moe_gate", "ec2moe_route", "ec2moe_experts", "ec2moe_shared_experts", "ec2moe_combine",
     "ec2moe_lr_encode", "ec2moe_lr_decode", "ec2moe_layer_forward", "ec2moe_last_device_error",
     "ec2moe_last_launch_count", "ec2moe_status_string", "ec2moe_profile_enable", "ec2moe_profile_count",
-    "ec2moe_profile_read", "ec2moe_profile_reset",
+    "ec2moe_profile_read", "ec2moe_profile_reset", "ec2moe_route_noalloc",
 ]
 
 
@@ -71,6 +71,7 @@ _SIGS = {
     "ec2moe_route_workspace_size": (ctypes.c_size_t, [_D]),
     "ec2moe_gate": (ctypes.c_int, [_D, _P, _P, _P, _P, _P, _P, _P, _P, _P]),
     "ec2moe_route": (ctypes.c_int, [_D, _P, _P, _P, _P, _P, _P, ctypes.c_int32, _P, _P, ctypes.c_size_t, _P]),
+    "ec2moe_route_noalloc": (ctypes.c_int, [_D, _P, _P, _P, _P, _P, _P, ctypes.c_int32, _P, _P]),
     "ec2moe_experts": (ctypes.c_int, [_D, _P, _P, _P, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "ec2moe_shared_experts": (ctypes.c_int, [_D, _P, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "ec2moe_combine": (ctypes.c_int, [_D, _P, _P, _P, _P]),
@@ -176,6 +177,14 @@ def ec2moe_route(desc, topk_idx, counts, offsets, perm, inv_perm=None, src=None,
     _check(load().ec2moe_route(_dref(desc), _ptr(topk_idx), _ptr(counts), _ptr(offsets), _ptr(perm),
                                _ptr(inv_perm), _ptr(src), int(width), _ptr(dst), _ptr(workspace), int(ws_bytes),
                                _stream(stream)), "ec2moe_route")
+
+
+def ec2moe_route_noalloc(desc, topk_idx, counts, offsets, perm, inv_perm=None, src=None, width=0, dst=None,
+                         stream=None):
+    """ec2moe_route without a workspace: the histograms use a fixed array inside the library."""
+    _check(load().ec2moe_route_noalloc(_dref(desc), _ptr(topk_idx), _ptr(counts), _ptr(offsets), _ptr(perm),
+                                       _ptr(inv_perm), _ptr(src), int(width), _ptr(dst), _stream(stream)),
+           "ec2moe_route_noalloc")
 
 
 def ec2moe_experts(desc, X_perm, offsets, W1, W3, W2, topk_w, perm, slot_out, workspace, ws_bytes, stream=None):
