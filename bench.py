@@ -11,7 +11,11 @@ rank-128 codec).
 Timing: W untimed warm-up steps, then K steps, each bracketed by CUDA events
 on the launching stream with L2 flushed (256 MiB write) between steps; a
 barrier and a device synchronise bracket the timed loop; the max over ranks is
-reported.  Under torchrun each rank runs its own batch (token-parallel
+reported.  ``value`` replays one ``ec2moe_layer_forward`` call captured in a
+CUDA graph (inputs resident in HBM); ``e2e`` calls the C ABI eagerly every step
+with the host<->device copies of X and y inside the timed region.  Per-kernel
+times come from CUDA events the library records around each of its launches
+(``ec2moe_profile_*``) inside a graph-captured call.  Under torchrun each rank runs its own batch (token-parallel
 replicas, no collective on the data path; weak scaling).
 
 ``--impl reference`` times the fp64 CPU oracle instead, on the host cores.
@@ -328,6 +332,28 @@ def run_ours(args):
         barrier()
         return [a.elapsed_time(b) for a, b in evs]
 
+    # One layer call captured in a CUDA graph: the same kernels with the host's
+    # launch overhead taken out of the device-resident measurement.
+    def capture(profile: bool):
+        if profile:
+            C.ec2moe_profile_reset()
+            C.ec2moe_profile_enable(True)
+            run.forward(stream=stream)  # fills the library's event pool outside capture
+            torch.cuda.synchronize(dev)
+            C.ec2moe_profile_reset()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            run.forward(stream=torch.cuda.current_stream(dev))
+        if profile:
+            C.ec2moe_profile_enable(False)
+        torch.cuda.synchronize(dev)
+        return g
+
+    graph = capture(False)
+    for _ in range(3):
+        graph.replay()
+    torch.cuda.synchronize(dev)
+
     clocks = None
     sampler = None
     if rank == 0:
@@ -339,14 +365,14 @@ def run_ours(args):
             time.sleep(0.3)
         except Exception:
             sampler = None
-    step_ms = timed_loop(lambda: run.forward(stream=stream))
+    step_ms = timed_loop(graph.replay)
     if sampler:
         clocks = sampler.stop()
     status = C.ec2moe_last_device_error(stream)
     if status != C.OK:
         raise RuntimeError(f"device error in the timed loop: {C.status_string(status)}")
 
-    # End to end through the public call: pinned host X -> device, layer, Y -> pinned host.
+    # End to end through the public call, eager: pinned host X -> device, layer, Y -> pinned host.
     X_host = inp["X"].to("cpu").pin_memory()
     Y_host = torch.empty(run.Y.shape, dtype=run.Y.dtype).pin_memory()
     X_dev = torch.empty_like(inp["X"])
@@ -360,20 +386,17 @@ def run_ours(args):
         e2e_step()
     e2e_ms = timed_loop(e2e_step)
 
-    # Per-kernel device time: the same steps with every launch bracketed by events.
-    C.ec2moe_profile_reset()
-    C.ec2moe_profile_enable(True)
+    # Per-kernel device time: every launch of the graphed call bracketed by events.
+    pgraph = capture(True)
     prof_steps = max(args.steps, 5)
-    barrier()
+    per_kernel = {}
     for _ in range(prof_steps):
         flush.zero_()
-        run.forward(stream=stream)
-    barrier()
-    C.ec2moe_profile_enable(False)
-    per_kernel = {}
-    for i in range(C.ec2moe_profile_count()):
-        name, ms = C.ec2moe_profile_read(i)
-        per_kernel.setdefault(name, []).append(ms)
+        pgraph.replay()
+        torch.cuda.synchronize(dev)
+        for i in range(C.ec2moe_profile_count()):
+            name, ms = C.ec2moe_profile_read(i)
+            per_kernel.setdefault(name, []).append(ms)
     C.ec2moe_profile_reset()
 
     total_ms = torch.tensor([sum(step_ms), sum(e2e_ms)], dtype=torch.float64, device=dev)
@@ -413,6 +436,7 @@ def run_ours(args):
         "warmup": args.warmup, "ms_per_step": round(t_step, 5), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if cfg.dtype == 1 else "f32", "data": "synthetic",
         "config": {"workload": describe(cfg), "l2": "flushed between steps (256 MiB write)",
+                   "launch": "value: CUDA graph of one ec2moe_layer_forward call; e2e: eager C-ABI call",
                    "parallelism": f"token-parallel replicas x{world}"},
         "layer_tflops": round(layer_flops / (t_step * 1e-3) / 1e12, 2),
         "layer_frac_bf16_peak": round(layer_flops / (t_step * 1e-3) / 1e12 / peaks["bf16_tflops"], 4),

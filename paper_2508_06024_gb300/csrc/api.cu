@@ -26,6 +26,16 @@ std::vector<ProfRecord> g_prof;
 std::vector<cudaEvent_t> g_pool;
 size_t g_pool_used = 0;
 
+// Records `e` on `s`; inside a stream capture the record becomes a graph node
+// (cudaEventRecordExternal), so timings survive graph replay.
+void record_on(cudaEvent_t e, cudaStream_t s) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+    cudaEventRecordWithFlags(e, s, cudaEventRecordExternal);
+  else
+    cudaEventRecord(e, s);
+}
+
 cudaEvent_t pool_event() {
   if (g_pool_used == g_pool.size()) {
     cudaEvent_t e = nullptr;
@@ -43,7 +53,7 @@ KernelScope::KernelScope(const char* name, cudaStream_t s) : name_(name), s_(s) 
   std::lock_guard<std::mutex> lock(g_prof_mu);
   if (g_prof_on) {
     start_ = pool_event();
-    if (start_) cudaEventRecord(start_, s_);
+    if (start_) record_on(start_, s_);
   }
 }
 
@@ -53,7 +63,7 @@ KernelScope::~KernelScope() {
   if (g_prof_on && start_) {
     cudaEvent_t stop = pool_event();
     if (stop) {
-      cudaEventRecord(stop, s_);
+      record_on(stop, s_);
       g_prof.push_back(ProfRecord{name_, start_, stop});
     }
   }
@@ -72,6 +82,31 @@ int sm_count() {
     cache[dev] = n;
   }
   return cache[dev];
+}
+
+cudaError_t ensure_smem_attr(const void* kernel, int bytes) {
+  struct Entry {
+    int dev;
+    const void* kernel;
+    int bytes;
+  };
+  static std::mutex mu;
+  static std::vector<Entry> set;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  for (Entry& en : set) {
+    if (en.dev == dev && en.kernel == kernel) {
+      if (en.bytes >= bytes) return cudaSuccess;
+      e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+      if (e == cudaSuccess) en.bytes = bytes;
+      return e;
+    }
+  }
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) set.push_back(Entry{dev, kernel, bytes});
+  return e;
 }
 
 }  // namespace ec2moe

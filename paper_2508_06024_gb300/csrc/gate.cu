@@ -233,6 +233,255 @@ __global__ void __launch_bounds__(WARPS * 32) gate_topk_kernel(const KParams p) 
   }
 }
 
+// Warp-cooperative decision for one token from its logits L[0..E) (local) and
+// L[E..E+K) (global) in shared memory.  Lane l owns experts l, l+32, l+64, l+96.
+// Same arithmetic as gate_topk_kernel: key = l_i (K = 1) or (m_k - lse_k) + l_i,
+// Top-k by k rounds of a warp argmax with ties to the lower index, weight
+// g_i = exp((m_k - LSE_m) + (l_i - lse_k)).
+__device__ void decide_token_warp(const KParams& p, const float* L, int tok, int lane) {
+  const int nglob = (p.K == 1) ? 0 : p.K;
+  const int gsize = p.E / p.K;
+  float lv[4];
+  bool al[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = lane + 32 * i;
+    al[i] = e < p.E && allowed_bit(p, e);
+    lv[i] = al[i] ? L[e] : -CUDART_INF_F;
+  }
+  float key[4], lw[4];
+  if (!nglob) {
+    // one group: warp max and warp sum of the allowed logits
+    float mx = fmaxf(fmaxf(lv[0], lv[1]), fmaxf(lv[2], lv[3]));
+#pragma unroll
+    for (int sh = 16; sh > 0; sh >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, sh));
+    float sum = 0.0f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (al[i]) sum += expf(lv[i] - mx);
+#pragma unroll
+    for (int sh = 16; sh > 0; sh >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, sh);
+    const float lse = mx + logf(sum);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      key[i] = lv[i];
+      lw[i] = lv[i] - lse;
+    }
+  } else {
+    // lane g < K: log-sum-exp of group g's allowed logits; then the group softmax
+    float lse_mine = -CUDART_INF_F;
+    if (lane < p.K) {
+      const int lo = lane * gsize;
+      float mx = -CUDART_INF_F;
+      for (int e = lo; e < lo + gsize; ++e)
+        if (allowed_bit(p, e)) mx = fmaxf(mx, L[e]);
+      float sum = 0.0f;
+      for (int e = lo; e < lo + gsize; ++e)
+        if (allowed_bit(p, e)) sum += expf(L[e] - mx);
+      if (mx > -CUDART_INF_F) lse_mine = mx + logf(sum);
+    }
+    const float mk_mine = (lane < p.K && lse_mine > -CUDART_INF_F) ? L[p.E + lane] : -CUDART_INF_F;
+    float mxm = mk_mine;
+#pragma unroll
+    for (int sh = 16; sh > 0; sh >>= 1) mxm = fmaxf(mxm, __shfl_xor_sync(0xffffffffu, mxm, sh));
+    float summ = (mk_mine > -CUDART_INF_F) ? expf(mk_mine - mxm) : 0.0f;
+#pragma unroll
+    for (int sh = 16; sh > 0; sh >>= 1) summ += __shfl_xor_sync(0xffffffffu, summ, sh);
+    const float lse_m = mxm + logf(summ);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int e = lane + 32 * i;
+      const int g = (e < p.E ? e : 0) / gsize;
+      const float lse_g = __shfl_sync(0xffffffffu, lse_mine, g);
+      const float mk = L[p.E + (g < p.K ? g : 0)];
+      key[i] = al[i] ? (mk - lse_g) + lv[i] : -CUDART_INF_F;
+      lw[i] = (mk - lse_m) + (lv[i] - lse_g);
+    }
+  }
+  float wsum = 0.0f, w_mine = 0.0f;
+  int id_mine = 0;
+  for (int s = 0; s < p.k; ++s) {
+    float bk = -CUDART_INF_F, bw = 0.0f;
+    int bi = 0x7fffffff;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int e = lane + 32 * i;
+      if (key[i] > -CUDART_INF_F && better(key[i], e, bk, bi)) {
+        bk = key[i];
+        bi = e;
+        bw = lw[i];
+      }
+    }
+#pragma unroll
+    for (int sh = 16; sh > 0; sh >>= 1) {
+      const float ok = __shfl_xor_sync(0xffffffffu, bk, sh);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, sh);
+      const float ow = __shfl_xor_sync(0xffffffffu, bw, sh);
+      if (better(ok, oi, bk, bi)) {
+        bk = ok;
+        bi = oi;
+        bw = ow;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (lane + 32 * i == bi) key[i] = -CUDART_INF_F;
+    const float g = expf(bw);
+    wsum += g;
+    if (lane == s) {
+      id_mine = bi;
+      w_mine = g;
+    }
+  }
+  if (lane < p.k) {
+    p.topk_idx[(size_t)tok * p.k + lane] = id_mine;
+    p.topk_w[(size_t)tok * p.k + lane] = p.renorm ? w_mine / wsum : w_mine;
+  }
+}
+
+// Gate with every gate row resident in shared memory.  A block of 256 threads
+// owns BT = TPT * 256 / S tokens at a time; thread (s, q) holds the slice
+// [s*SW, (s+1)*SW) of d_model of TPT tokens in registers (all loads issued
+// before the first FMA) and accumulates their dot products with up to NB gate
+// rows, so every 16-byte weight load from shared memory (a broadcast shared by
+// the threads of a slice) feeds 4*TPT FMAs.  Slice partials go to shared
+// memory in an [n][slice][token] layout padded so both the writes and the
+// fixed-order sums over slices are free of bank conflicts; one warp per token
+// then takes the softmax / Top-k decision.
+constexpr int SL_THREADS = 256;
+constexpr int SL_RED_PAD = 16;
+
+// Raw 16-byte vectors of one 8-element activation chunk (bf16: one, fp32: two).
+template <typename TX>
+struct Chunk8 {
+  static constexpr int NV = sizeof(TX) == 2 ? 1 : 2;
+  U4 v[NV];
+  __device__ __forceinline__ void load(const TX* p) {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) v[i] = reinterpret_cast<const U4*>(p)[i];
+  }
+  __device__ __forceinline__ void zero() {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) v[i] = U4{0u, 0u, 0u, 0u};
+  }
+  __device__ __forceinline__ void to_float(float* f) const {
+    if (NV == 1) {
+      f[0] = bf16_lo(v[0].x); f[1] = bf16_hi(v[0].x); f[2] = bf16_lo(v[0].y); f[3] = bf16_hi(v[0].y);
+      f[4] = bf16_lo(v[0].z); f[5] = bf16_hi(v[0].z); f[6] = bf16_lo(v[0].w); f[7] = bf16_hi(v[0].w);
+    } else {
+#pragma unroll
+      for (int i = 0; i < NV; ++i) {
+        f[4 * i + 0] = __uint_as_float(v[i].x); f[4 * i + 1] = __uint_as_float(v[i].y);
+        f[4 * i + 2] = __uint_as_float(v[i].z); f[4 * i + 3] = __uint_as_float(v[i].w);
+      }
+    }
+  }
+};
+
+template <typename TX, int XC, int TPT, int NB>
+__global__ void __launch_bounds__(SL_THREADS) gate_slices_kernel(const KParams p, int S) {
+  extern __shared__ float smem_f[];
+  const int nglob = (p.K == 1) ? 0 : p.K;
+  const int O = p.E + nglob;
+  const int JQ = SL_THREADS / S;       // token groups per tile
+  const int BT = JQ * TPT;             // tokens per tile
+  const int SW = p.d / S;
+  const int nch = SW / 8;
+  const int RS = S * BT + SL_RED_PAD;  // row stride of the partials
+  float* sW = smem_f;                   // [O][d]
+  float* sRed = sW + (size_t)O * p.d;   // [NB][RS]
+  float* sLog = sRed + NB * RS;         // [BT][O]
+  const int jq = threadIdx.x % JQ;
+  const int sl = threadIdx.x / JQ;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  {  // stage the gate rows, eight 16-byte loads in flight per thread
+    const int n4 = O * p.d / 4;
+    float4* dst = reinterpret_cast<float4*>(sW);
+    const int e4 = p.E * p.d / 4;
+    for (int base = threadIdx.x; base < n4; base += SL_THREADS * 8) {
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = base + u * SL_THREADS;
+        if (i < n4)
+          v[u] = i < e4 ? reinterpret_cast<const float4*>(p.W_local)[i]
+                        : reinterpret_cast<const float4*>(p.W_global)[i - e4];
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = base + u * SL_THREADS;
+        if (i < n4) dst[i] = v[u];
+      }
+    }
+  }
+  __syncthreads();
+
+  const TX* X = reinterpret_cast<const TX*>(p.X);
+  const int n_tiles = (p.T + BT - 1) / BT;
+  for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    Chunk8<TX> xs[TPT][XC];
+#pragma unroll
+    for (int t = 0; t < TPT; ++t) {
+      const int tok = tile * BT + jq * TPT + t;
+#pragma unroll
+      for (int c = 0; c < XC; ++c) {
+        if (c < nch && tok < p.T) xs[t][c].load(X + (size_t)tok * p.d + sl * SW + c * 8);
+        else xs[t][c].zero();
+      }
+    }
+    for (int ob = 0; ob < O; ob += NB) {
+      float acc[TPT][NB];
+#pragma unroll
+      for (int t = 0; t < TPT; ++t)
+#pragma unroll
+        for (int n = 0; n < NB; ++n) acc[t][n] = 0.0f;
+#pragma unroll
+      for (int c = 0; c < XC; ++c) {
+        if (c < nch) {
+          float xf[TPT][8];
+#pragma unroll
+          for (int t = 0; t < TPT; ++t) xs[t][c].to_float(xf[t]);
+          const float* wcol = sW + sl * SW + c * 8;
+#pragma unroll
+          for (int n = 0; n < NB; ++n) {
+            if (ob + n < O) {
+              float wv[8];
+              load8(wcol + (size_t)(ob + n) * p.d, wv);
+#pragma unroll
+              for (int t = 0; t < TPT; ++t)
+#pragma unroll
+                for (int q = 0; q < 8; ++q) acc[t][n] = fmaf(xf[t][q], wv[q], acc[t][n]);
+            }
+          }
+        }
+      }
+#pragma unroll
+      for (int n = 0; n < NB; ++n) {
+        float* dst = sRed + n * RS + sl * BT + jq * TPT;
+        if (TPT == 2) *reinterpret_cast<float2*>(dst) = make_float2(acc[0][n], acc[TPT - 1][n]);
+        else dst[0] = acc[0][n];
+      }
+      __syncthreads();
+      for (int i = threadIdx.x; i < BT * NB; i += SL_THREADS) {
+        const int n = i / BT, jj = i % BT;
+        const int o = ob + n;
+        if (o < O) {
+          float sum = 0.0f;
+          for (int q = 0; q < S; ++q) sum += sRed[n * RS + q * BT + jj];
+          sLog[jj * O + o] = sum + (o < p.E ? p.b_local[o] : p.b_global[o - p.E]);
+        }
+      }
+      __syncthreads();
+    }
+    for (int jj = warp; jj < BT; jj += SL_THREADS / 32) {
+      const int tok = tile * BT + jj;
+      if (tok < p.T) decide_token_warp(p, sLog + jj * O, tok, lane);
+    }
+    __syncthreads();
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
@@ -252,6 +501,54 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
   p.topk_idx = a.topk_idx;
   p.topk_w = a.topk_w;
   const int O = a.E + (a.K == 1 ? 0 : a.K);
+  cudaError_t e;
+  // Slice kernel when every gate row fits in shared memory next to the
+  // partials: S slices of d_model per token (SW = d / S <= 128, a multiple of
+  // 8), two tokens per thread while the slice is at most 64 wide, preferring
+  // enough token tiles to give every SM two.
+  {
+    int S = 0, TPT = 2;
+    for (int cand : {8, 16, 32}) {
+      if (a.d % (8 * cand) != 0 || a.d / cand > 128) continue;
+      S = cand;
+      TPT = (a.d / cand <= 64) ? 2 : 1;
+      const long long bt = (long long)(SL_THREADS / cand) * TPT;
+      if ((a.T + bt - 1) / bt >= 2LL * sm_count()) break;
+    }
+    const int NB = O <= 16 ? 16 : 32;
+    const int BT = S ? (SL_THREADS / S) * TPT : 0;
+    const size_t smem = (size_t)O * a.d * 4 + (size_t)NB * (S * BT + SL_RED_PAD) * 4 + (size_t)BT * O * 4;
+    if (S && smem <= 160 * 1024) {
+      const long long tiles = (a.T + BT - 1) / BT;
+      const int per_sm = smem <= 72 * 1024 ? 3 : (smem <= 110 * 1024 ? 2 : 1);
+      long long blocks = tiles < (long long)sm_count() * per_sm ? tiles : (long long)sm_count() * per_sm;
+      if (blocks < 1) blocks = 1;
+      const int nch = a.d / S / 8;
+      KernelScope ks("gate_topk", s);
+#define EC2MOE_SLICES(TX, XC, TP, NBV)                                                                       \
+  do {                                                                                                      \
+    e = ensure_smem_attr(reinterpret_cast<const void*>(gate_slices_kernel<TX, XC, TP, NBV>), (int)smem);     \
+    if (e != cudaSuccess) return e;                                                                         \
+    gate_slices_kernel<TX, XC, TP, NBV><<<(int)blocks, SL_THREADS, smem, s>>>(p, S);                        \
+  } while (0)
+#define EC2MOE_SLICES_NB(TX, XC, TP) \
+  do {                               \
+    if (NB == 16) EC2MOE_SLICES(TX, XC, TP, 16); else EC2MOE_SLICES(TX, XC, TP, 32); \
+  } while (0)
+      if (bf16) {
+        if (nch <= 4) EC2MOE_SLICES_NB(__nv_bfloat16, 4, 2);
+        else if (nch <= 8) EC2MOE_SLICES_NB(__nv_bfloat16, 8, 2);
+        else EC2MOE_SLICES_NB(__nv_bfloat16, 16, 1);
+      } else {
+        if (nch <= 4) EC2MOE_SLICES_NB(float, 4, 2);
+        else if (nch <= 8) EC2MOE_SLICES_NB(float, 8, 2);
+        else EC2MOE_SLICES_NB(float, 16, 1);
+      }
+#undef EC2MOE_SLICES_NB
+#undef EC2MOE_SLICES
+      return cudaGetLastError();
+    }
+  }
   const size_t base = (size_t)(WARPS * TPW * MAXO + WARPS * TPW * 32) * sizeof(float);
   const size_t wbytes = (size_t)O * a.d * sizeof(float);
   const bool w_smem = base + wbytes <= 200 * 1024;
@@ -263,11 +560,10 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
   const int cap = w_smem ? sm_count() : sm_count() * 4;
   if (blocks > cap) blocks = cap;
   if (blocks < 1) blocks = 1;
-  cudaError_t e;
   KernelScope ks("gate_topk", s);
 #define EC2MOE_GATE_LAUNCH(TX, WS)                                                                          \
   do {                                                                                                      \
-    e = cudaFuncSetAttribute(gate_topk_kernel<TX, WS>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+    e = ensure_smem_attr(reinterpret_cast<const void*>(gate_topk_kernel<TX, WS>), (int)smem);            \
     if (e != cudaSuccess) return e;                                                                         \
     gate_topk_kernel<TX, WS><<<blocks, WARPS * 32, smem, s>>>(p);                                           \
   } while (0)

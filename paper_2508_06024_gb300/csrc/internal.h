@@ -29,6 +29,10 @@ class KernelScope {
 
 int sm_count();
 
+// cudaFuncSetAttribute(MaxDynamicSharedMemorySize) once per (device, kernel),
+// raised only when a launch needs more than was set before.
+cudaError_t ensure_smem_attr(const void* kernel, int bytes);
+
 // ----------------------------------------------------------------- gate (Eq. 4-7)
 struct GateArgs {
   const void* X;  // [T, d] bf16 or fp32

@@ -9,11 +9,12 @@
 // step-specific op (plain store, GELU, SwiGLU, or gate-scale + scatter to the
 // token's slot for the combine of Eq. 1).
 //
-// CTA layout (192 threads):
+// CTA layout (320 threads):
 //   warp 0      TMA producer (one elected lane)
 //   warp 1      TMEM allocator + MMA issuer (one elected lane)
-//   warps 2..5  epilogue: TMEM -> registers -> global (warp w reads TMEM lanes
-//               32*(w%4) .. +31, i.e. rows of the 128-row tile)
+//   warps 2..9  epilogue: TMEM -> registers -> global.  Warp w may only read
+//               TMEM lanes 32*(w%4) .. +31 (rows of the 128-row tile); the two
+//               warps of a lane quadrant split the tile's columns in halves.
 // Pipelines: STAGES shared-memory stages (full/empty mbarriers) and two TMEM
 // accumulators (tmem_full/tmem_empty) so the epilogue of tile i overlaps the
 // main loop of tile i+1.
@@ -41,7 +42,8 @@ namespace {
 constexpr int BM = 128;   // tile rows (MMA M, TMEM lanes)
 constexpr int BK = 64;    // K per stage: one 128-byte swizzle row of bf16
 constexpr int UK = 16;    // K of one tcgen05.mma kind::f16
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 320;
+constexpr int EPI_WARPS = 8;
 constexpr int MAX_GROUPS = 136;
 
 struct Params {
@@ -167,6 +169,24 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+template <int CW>
+__device__ __forceinline__ void tmem_ld(uint32_t taddr, float* v) {
+  if (CW == 32) tmem_ld32(taddr, v);
+  else tmem_ld16(taddr, v);
+}
+
 // ------------------------------------------------------------------ tile schedule
 struct TileCoord {
   int g, m_blk, n_blk;
@@ -181,13 +201,18 @@ __device__ __forceinline__ TileCoord decode_tile(int tile, const int* tile_prefi
   return TileCoord{cursor, rem % mt, rem / mt};
 }
 
+constexpr int pow2_at_least(int x) { return x <= 32 ? 32 : (x <= 64 ? 64 : (x <= 128 ? 128 : (x <= 256 ? 256 : 512))); }
+
 template <int BN, int EPI, int STAGES>
 struct Cfg {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int BN_OUT = (EPI == EPI_SWIGLU) ? BN / 2 : BN;
-  static constexpr int TMEM_COLS = 2 * BN;  // two accumulators
+  static constexpr int HALF = BN_OUT / 2;               // columns per epilogue warp
+  static constexpr int CW = (HALF % 32 == 0) ? 32 : 16;  // columns per TMEM load (divides HALF)
+  static_assert(HALF % CW == 0 && CW % 16 == 0, "epilogue chunks must tile each half exactly");
+  static constexpr int TMEM_COLS = pow2_at_least(2 * BN);  // two accumulators
   static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8;
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES + 16 + 2 * (MAX_GROUPS + 1) * 4;
 };
@@ -222,7 +247,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), 4);
+      mbar_init(smem_u32(&tempty[a]), EPI_WARPS);
     }
     mbar_init(smem_u32(drain), 1);
     *abort_flag = 0;
@@ -356,7 +381,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // ---------------------------------------------------------------- epilogue
-    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    const int q = warp & 3;          // TMEM lane quadrant this warp may access
+    const int half = (warp - 2) >> 2;  // which half of the tile's columns
     const int row_in_tile = q * 32 + lane;
     int it = 0;
     int cursor = 0;
@@ -379,25 +405,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t t_row = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
       __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out) + dest * p.ldo;
 #pragma unroll 1
-      for (int c0 = 0; c0 < C::BN_OUT; c0 += 32) {
+      for (int c0 = half * C::HALF; c0 < (half + 1) * C::HALF; c0 += C::CW) {
         const int col = tc.n_blk * C::BN_OUT + c0;
-        float v[32];
-        tmem_ld32(t_row + c0, v);
+        float v[C::CW];
+        tmem_ld<C::CW>(t_row + c0, v);
         if (EPI == EPI_SWIGLU) {
-          float u[32];
-          tmem_ld32(t_row + c0 + BN / 2, u);
+          float u[C::CW];
+          tmem_ld<C::CW>(t_row + c0 + BN / 2, u);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = silu(v[i]) * u[i];
+          for (int i = 0; i < C::CW; ++i) v[i] = silu(v[i]) * u[i];
         } else if (EPI == EPI_GELU) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = gelu_erf(v[i]);
+          for (int i = 0; i < C::CW; ++i) v[i] = gelu_erf(v[i]);
         } else if (EPI == EPI_SCATTER) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] *= sc;
+          for (int i = 0; i < C::CW; ++i) v[i] *= sc;
         }
         if (valid && col < p.N) {
 #pragma unroll
-          for (int j = 0; j < 4; ++j) store8(orow + col + 8 * j, v + 8 * j);
+          for (int j = 0; j < C::CW / 8; ++j) store8(orow + col + 8 * j, v + 8 * j);
         }
       }
       tc_fence_before();
@@ -430,9 +456,51 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
+bool encode_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows);
+
+// Encoded tensor maps are cached by (device, address, shape, box): encoding
+// costs host time on every launch otherwise.  A map only describes an address
+// and a layout, so a hit stays valid even if the memory was reallocated.
+struct MapKey {
+  int dev;
+  const void* ptr;
+  long long rows, cols;
+  int box_rows;
+  bool operator==(const MapKey& o) const {
+    return dev == o.dev && ptr == o.ptr && rows == o.rows && cols == o.cols && box_rows == o.box_rows;
+  }
+};
+
 // 2-D bf16 tensor map over a row-major [rows, cols] matrix, box = 64 columns x box_rows
 // rows, 128-byte swizzle, zero fill out of bounds.
 bool make_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+  constexpr int SLOTS = 64;
+  static std::mutex mu;
+  static MapKey keys[SLOTS];
+  static CUtensorMap maps[SLOTS];
+  static bool used[SLOTS] = {};
+  static int next = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  const MapKey key{dev, ptr, rows, cols, box_rows};
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < SLOTS; ++i)
+      if (used[i] && keys[i] == key) {
+        *m = maps[i];
+        return true;
+      }
+  }
+  if (!encode_map(m, ptr, rows, cols, box_rows)) return false;
+  std::lock_guard<std::mutex> lock(mu);
+  keys[next] = key;
+  maps[next] = *m;
+  used[next] = true;
+  next = (next + 1) % SLOTS;
+  return true;
+}
+
+bool encode_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
   auto fn = encode_fn();
   if (!fn) return false;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
@@ -457,12 +525,7 @@ const char* kernel_name(int epi) {
 template <int BN, int EPI, int STAGES>
 cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   using C = Cfg<BN, EPI, STAGES>;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(tc_gemm_kernel<BN, EPI, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    C::SMEM);
-  });
+  cudaError_t attr_err = ensure_smem_attr(reinterpret_cast<const void*>(tc_gemm_kernel<BN, EPI, STAGES>), C::SMEM);
   if (attr_err != cudaSuccess) return attr_err;
   CUtensorMap mA, mB, mB2;
   const int b_box = (EPI == EPI_SWIGLU) ? BN / 2 : BN;
@@ -498,21 +561,53 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+// Smem budget of the operand pipeline: as many stages as fit in ~200 KB.
+constexpr int stages_for(int bn) { return (200 * 1024) / (BM * BK * 2 + bn * BK * 2) > 8 ? 8 : (200 * 1024) / (BM * BK * 2 + bn * BK * 2); }
+
+template <int EPI>
+cudaError_t launch_epi(const GemmArgs& a, int bn, cudaStream_t s) {
+  switch (bn) {
+    case 32:
+      if constexpr (EPI != EPI_SWIGLU) return launch_cfg<32, EPI, stages_for(32)>(a, s);
+      break;
+    case 64: return launch_cfg<64, EPI, stages_for(64)>(a, s);
+    case 128: return launch_cfg<128, EPI, stages_for(128)>(a, s);
+    case 192: return launch_cfg<192, EPI, stages_for(192)>(a, s);
+    case 256: return launch_cfg<256, EPI, stages_for(256)>(a, s);
+  }
+  return cudaErrorInvalidValue;
+}
+
+// N-tile choice: the widest tile whose expected tile count still gives every
+// SM work (>= 90% of the SMs), else the narrowest (most parallel) tile.  The
+// m-tile count of a grouped GEMM is only known on the device; half a partial
+// tile per group is expected.
+int choose_bn(const GemmArgs& a, int epi) {
+  const double m_tiles = (double)a.max_rows / BM + (a.G > 1 ? 0.5 * a.G : 0.0) + (a.G == 1 && a.max_rows % BM ? 1 : 0);
+  const int sms = sm_count();
+  const int cands[5] = {256, 192, 128, 64, 32};
+  int pick = 0;
+  for (int bn : cands) {
+    const int out = (epi == EPI_SWIGLU) ? bn / 2 : bn;
+    if (epi == EPI_SWIGLU && bn < 64) continue;
+    if (out > a.N && bn != 32 && !(epi == EPI_SWIGLU && bn == 64)) continue;  // no wider than N
+    pick = bn;
+    const double tiles = m_tiles * ((a.N + out - 1) / out);
+    if (tiles >= 0.9 * sms) return bn;
+  }
+  return pick;
+}
+
 }  // namespace
 
 cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
   if (a.G < 1 || a.G > MAX_GROUPS || a.N % 32 != 0 || a.K % 8 != 0) return cudaErrorInvalidValue;
-  // Wide N tiles where N allows it; 128 otherwise.
-  const bool wide = (epi == EPI_SWIGLU) ? (a.N % 128 == 0) : (a.N % 256 == 0);
+  const int bn = choose_bn(a, epi);
   switch (epi) {
-    case EPI_STORE:
-      return wide ? launch_cfg<256, EPI_STORE, 4>(a, s) : launch_cfg<128, EPI_STORE, 6>(a, s);
-    case EPI_GELU:
-      return wide ? launch_cfg<256, EPI_GELU, 4>(a, s) : launch_cfg<128, EPI_GELU, 6>(a, s);
-    case EPI_SWIGLU:
-      return wide ? launch_cfg<256, EPI_SWIGLU, 4>(a, s) : launch_cfg<128, EPI_SWIGLU, 6>(a, s);
-    case EPI_SCATTER:
-      return wide ? launch_cfg<256, EPI_SCATTER, 4>(a, s) : launch_cfg<128, EPI_SCATTER, 6>(a, s);
+    case EPI_STORE: return launch_epi<EPI_STORE>(a, bn, s);
+    case EPI_GELU: return launch_epi<EPI_GELU>(a, bn, s);
+    case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, s);
+    case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, s);
   }
   return cudaErrorInvalidValue;
 }

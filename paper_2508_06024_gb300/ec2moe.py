@@ -124,8 +124,8 @@ def _stream(stream) -> Optional[int]:
 
 
 def _mask(mask):
-    if mask is None:
-        return None
+    if mask is None or isinstance(mask, ctypes.Array):
+        return mask
     vals = [int(v) for v in (mask.tolist() if hasattr(mask, "tolist") else mask)]
     return (ctypes.c_uint8 * len(vals))(*vals)
 
@@ -146,6 +146,11 @@ def status_string(status: int) -> str:
 def make_desc(T, d, E, d_ff, k, n_groups=1, act=GELU, dtype=BF16, r=0, n_shared=0, d_ff_shared=0,
               renorm_topk=0) -> LayerDesc:
     return LayerDesc(T, d, E, d_ff, k, n_groups, act, dtype, r, n_shared, d_ff_shared, renorm_topk)
+
+
+def host_mask(mask):
+    """A reusable host uint8 array for the ``mask`` argument (saves per-call marshalling)."""
+    return _mask(mask)
 
 
 def make_weights(W_local=None, b_local=None, W_global=None, b_global=None, W1=None, W3=None, W2=None,

@@ -35,7 +35,7 @@ class LayerRun:
         self.inp = inp
         self.desc = desc_for(cfg)
         self.weights = weights_for(inp)
-        self.mask = inp["mask"].to("cpu")
+        self.mask = C.host_mask(inp["mask"].to("cpu"))
         dt = cfg.torch_dtype
         T = cfg.T
         self.Y = torch.empty(T, cfg.d, dtype=dt, device=device)
