@@ -113,8 +113,8 @@ def kernel_work(cfg, name: str):
         return 0.0, 2 * es * n * d + 4 * n
     if name == "combine":
         return 0.0, es * (n * d + cfg.n_shared * T * d + T * d)
-    if name in ("route_count", "route_scatter"):
-        return 0.0, 4 * n * (1 if name == "route_count" else 3)
+    if name in ("route_count", "route_scatter", "route"):
+        return 0.0, 4 * n * {"route_count": 1, "route_scatter": 3, "route": 4}[name]
     return 0.0, 0.0
 
 

@@ -3,10 +3,12 @@
 // EC^2MoE MoE-layer forward.
 #include <cuda_runtime.h>
 
+#include <stdlib.h>
+
 #include <mutex>
 #include <vector>
 
-#include "../../include/ec2moe.h"
+#include "ec2moe.h"
 #include "internal.h"
 
 namespace ec2moe {
@@ -47,6 +49,14 @@ cudaEvent_t pool_event() {
 }  // namespace
 
 void reset_launch_count() { t_launches = 0; }
+
+bool next_launch_pdl() {
+  static const bool disabled = [] {
+    const char* v = getenv("EC2MOE_NO_PDL");
+    return v && v[0] == '1';
+  }();
+  return !disabled && t_launches > 0;
+}
 int launch_count() { return t_launches; }
 
 KernelScope::KernelScope(const char* name, cudaStream_t s) : name_(name), s_(s) {
@@ -213,6 +223,7 @@ LayerWs layer_ws(const ec2moe_layer_desc* d) {
 GemmArgs gemm_base() {
   GemmArgs g{};
   g.timeout_cycles = default_timeout_cycles();
+  g.self_row_base = -1;
   return g;
 }
 
@@ -227,7 +238,7 @@ cudaError_t run_gemm(const ec2moe_layer_desc* d, const GemmArgs& g, int epi, cud
 cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long long a_rows, long long a_row_base,
                     const int32_t* offsets, const void* W1, const void* W3, const void* W2, void* H, long long h_rows,
                     long long h_row_base, const int32_t* perm, const float* scale, void* out, long long out_row_base,
-                    cudaStream_t s) {
+                    cudaStream_t s, int g_active = 0) {
   const int ff = routed ? d->d_ff : d->d_ff_shared;
   const int G = routed ? d->E : d->n_shared;
   const long long rows = routed ? (long long)d->T * d->k : (long long)d->T * d->n_shared;
@@ -251,6 +262,7 @@ cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long
   up.out = H;
   up.ldo = ff;
   up.max_rows = rows;
+  up.g_active = routed ? g_active : 0;
   cudaError_t e = run_gemm(d, up, act_epi, s);
   if (e != cudaSuccess) return e;
   GemmArgs dn = gemm_base();
@@ -274,11 +286,23 @@ cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long
   dn.perm = routed ? perm : nullptr;
   dn.scale = routed ? scale : nullptr;
   dn.max_rows = rows;
+  dn.g_active = routed ? g_active : 0;
   return run_gemm(d, dn, routed ? EPI_SCATTER : EPI_STORE, s);
 }
 
+// Codec GEMM.  With `inv_perm` (decode only), row t of X_hat is written to
+// rows inv_perm[t*k + s] (s < k) of `out` -- the expert-ordered activations --
+// and, when self_row_base >= 0, also to row self_row_base + t.
+struct RelPlace {  // relative placement of decoded rows (routing fused into the gate)
+  const int32_t* counts = nullptr;
+  const int32_t* idx = nullptr;
+  int32_t* perm_out = nullptr;
+  int32_t* offsets_out = nullptr;
+};
+
 cudaError_t run_codec(const ec2moe_layer_desc* d, bool encode, const void* in, const void* V, void* out,
-                      cudaStream_t s) {
+                      cudaStream_t s, const int32_t* inv_perm = nullptr, long long self_row_base = -1,
+                      const RelPlace& rel = RelPlace()) {
   GemmArgs g = gemm_base();
   g.name = encode ? "lr_encode" : "lr_decode";
   g.A = in;
@@ -293,6 +317,17 @@ cudaError_t run_codec(const ec2moe_layer_desc* d, bool encode, const void* in, c
   g.out = out;
   g.ldo = g.N;
   g.max_rows = d->T;
+  if (inv_perm) {
+    g.perm = inv_perm;
+    g.rep_k = d->k;
+    g.self_row_base = self_row_base;
+    g.rep_counts = rel.counts;
+    g.rep_idx = rel.idx;
+    g.rep_perm_out = rel.perm_out;
+    g.rep_offsets_out = rel.offsets_out;
+    g.rep_E = d->E;
+    return run_gemm(d, g, EPI_REPLICATE, s);
+  }
   return run_gemm(d, g, EPI_STORE, s);
 }
 
@@ -565,24 +600,51 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   ga.renorm = desc->renorm_topk;
   ga.topk_idx = topk_idx;
   ga.topk_w = topk_w;
-  EC2MOE_CUDA(launch_gate(ga, bf, stream));
-  // Step 3b: routing tables.
-  EC2MOE_CUDA(launch_route(topk_idx, n, desc->E, blk, counts, offsets, perm, inv_perm, stream));
-  // Step 6: encode at the end, decode in the cloud (experts read X_hat).
+  // bf16 layers route inside the gate kernel (per-tile row reservations); the
+  // decoder (or the gather) then places rows and writes perm and offsets.
+  if (bf) {
+    ga.route_counts = counts;
+    ga.route_rel = inv_perm;
+  }
+  bool routed = false;
+  EC2MOE_CUDA(launch_gate(ga, bf, stream, &routed));
+  // Step 3b: routing tables (inside the gate kernel when it could take them).
+  if (!routed) EC2MOE_CUDA(launch_route(topk_idx, n, desc->E, blk, counts, offsets, perm, inv_perm, stream));
+  RelPlace rel;
+  if (routed) {
+    rel.counts = counts;
+    rel.idx = topk_idx;
+    rel.perm_out = perm;
+    rel.offsets_out = offsets;
+  }
+  // Step 6: encode at the end; decode in the cloud straight into expert order
+  // (the decoder's epilogue writes each X_hat row to its (token, slot)
+  // positions, and to the tail rows the shared experts read).
+  const void* shared_a = xa;
+  long long shared_a_rows = n + T, shared_a_base = n;
   if (desc->r > 0) {
     EC2MOE_CUDA(run_codec(desc, true, X, w->V_enc, zbuf, stream));
-    EC2MOE_CUDA(run_codec(desc, false, zbuf, w->V_dec, x_hat, stream));
+    EC2MOE_CUDA(run_codec(desc, false, zbuf, w->V_dec, xa, stream, inv_perm, desc->n_shared > 0 ? n : -1, rel));
   } else {
-    EC2MOE_CUDA(cudaMemcpyAsync(x_hat, X, (size_t)T * desc->d * es, cudaMemcpyDeviceToDevice, stream));
+    // Step 3b (move): rows of X into expert order; shared experts read X itself.
+    if (routed)
+      EC2MOE_CUDA(launch_gather_rel(X, xa, topk_idx, counts, inv_perm, perm, offsets, desc->E, n, desc->k, desc->d, bf,
+                                    stream));
+    else
+      EC2MOE_CUDA(launch_gather(X, xa, perm, n, desc->k, desc->d, bf, stream));
+    shared_a = X;
+    shared_a_rows = T;
+    shared_a_base = 0;
   }
-  // Step 3b (move): rows into expert order.
-  EC2MOE_CUDA(launch_gather(x_hat, xa, perm, n, desc->k, desc->d, bf, stream));
+  (void)x_hat;
   // Steps 4-5a: routed experts, gate scale and unpermute fused in the down projection.
+  int n_allowed = 0;
+  for (int e = 0; e < desc->E; ++e) n_allowed += mask[e] ? 1 : 0;
   EC2MOE_CUDA(run_ffn(desc, true, xa, n + T, 0, offsets, w->W1, w->W3, w->W2, h, n + (long long)desc->n_shared * T, 0,
-                      perm, topk_w, slot, 0, stream));
+                      perm, topk_w, slot, 0, stream, n_allowed));
   // Always-on shared experts on X_hat.
   if (desc->n_shared > 0) {
-    EC2MOE_CUDA(run_ffn(desc, false, xa, n + T, n, nullptr, w->W1s, w->W3s, w->W2s, h,
+    EC2MOE_CUDA(run_ffn(desc, false, shared_a, shared_a_rows, shared_a_base, nullptr, w->W1s, w->W3s, w->W2s, h,
                         n + (long long)desc->n_shared * T, n, nullptr, nullptr, shared, 0, stream));
   }
   // Step 5b: fixed-order combine (skipped when the down projection wrote Y directly).

@@ -9,6 +9,12 @@ namespace ec2moe {
 
 struct alignas(16) U4 { uint32_t x, y, z, w; };
 
+// Programmatic dependent launch: let the next kernel in the stream start its
+// independent prologue now / wait until the previous kernel's results are
+// complete and visible (a no-op when launched without the attribute).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xFFFF0000u); }
 
@@ -42,5 +48,27 @@ __device__ __forceinline__ void store8(float* p, const float* v) {
 __device__ __forceinline__ float gelu_erf(float u) { return 0.5f * u * (1.0f + erff(u * 0.70710678118654752f)); }
 // SiLU(u) = u / (1 + e^-u).
 __device__ __forceinline__ float silu(float u) { return u / (1.0f + expf(-u)); }
+
+// GELU for epilogues whose output is rounded to bf16 (relative step 2^-8).
+// erf(z), z >= 0, by formula 7.1.26 of Abramowitz & Stegun (Hastings):
+//   erf(z) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5)))) exp(-z^2),
+//   t = 1 / (1 + p z),  |error| <= 1.5e-7,
+// with erf odd for z < 0; exp and the reciprocal use the fast hardware paths
+// (relative error ~1e-7).  The GELU error is then below 2e-7 |u|, far under
+// the bf16 rounding of the result.
+__device__ __forceinline__ float gelu_bf16out(float u) {
+  const float z = fabsf(u) * 0.70710678118654752f;
+  const float t = __fdividef(1.0f, fmaf(0.3275911f, z, 1.0f));
+  float poly = fmaf(t, 1.061405429f, -1.453152027f);
+  poly = fmaf(t, poly, 1.421413741f);
+  poly = fmaf(t, poly, -0.284496736f);
+  poly = fmaf(t, poly, 0.254829592f);
+  poly *= t;
+  const float erf_abs = fmaf(-poly, __expf(-z * z), 1.0f);
+  return 0.5f * u * (1.0f + copysignf(erf_abs, u));
+}
+
+// SiLU for bf16-output epilogues: fast exp and division (relative error ~1e-7).
+__device__ __forceinline__ float silu_bf16out(float u) { return __fdividef(u, 1.0f + __expf(-u)); }
 
 }  // namespace ec2moe

@@ -41,6 +41,8 @@ struct KParams {
   int T, d, E, K, k, renorm;
   int32_t* topk_idx;
   float* topk_w;
+  int32_t* route_counts;  // fused routing: per-expert row counters (zero at launch); nullptr = gate only
+  int32_t* route_rel;     // fused routing: [T*k] row of each entry relative to its expert's first row
 };
 
 __device__ __forceinline__ bool allowed_bit(const KParams& p, int e) { return (p.mask_bits[e >> 5] >> (e & 31)) & 1u; }
@@ -58,6 +60,8 @@ __global__ void __launch_bounds__(WARPS * 32) gate_topk_kernel(const KParams p) 
   float* sGrp = sLog + WARPS * TPW * MAXO;              // [WARPS][TPW][2 * 16]: lse_k, then live flag
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  pdl_trigger();
+  pdl_wait();
 
   if (W_SMEM) {
     const int n4 = O * p.d / 4;
@@ -238,7 +242,7 @@ __global__ void __launch_bounds__(WARPS * 32) gate_topk_kernel(const KParams p) 
 // Same arithmetic as gate_topk_kernel: key = l_i (K = 1) or (m_k - lse_k) + l_i,
 // Top-k by k rounds of a warp argmax with ties to the lower index, weight
 // g_i = exp((m_k - LSE_m) + (l_i - lse_k)).
-__device__ void decide_token_warp(const KParams& p, const float* L, int tok, int lane) {
+__device__ void decide_token_warp(const KParams& p, const float* L, int tok, int lane, int* s_idx) {
   const int nglob = (p.K == 1) ? 0 : p.K;
   const int gsize = p.E / p.K;
   float lv[4];
@@ -336,6 +340,7 @@ __device__ void decide_token_warp(const KParams& p, const float* L, int tok, int
   if (lane < p.k) {
     p.topk_idx[(size_t)tok * p.k + lane] = id_mine;
     p.topk_w[(size_t)tok * p.k + lane] = p.renorm ? w_mine / wsum : w_mine;
+    if (s_idx) s_idx[lane] = id_mine;
   }
 }
 
@@ -378,6 +383,36 @@ struct Chunk8 {
   }
 };
 
+// ---- routing fused into the gate (layer path)
+// For each tile of BT tokens (nt = BT * k consecutive (token, slot) entries),
+// every expert present in the tile reserves a contiguous run of its rows with
+// one atomicAdd on route_counts[e] (zero at launch), and each entry's row
+// relative to its expert's first row -- the reserved base plus the entry's
+// stable rank among the tile's entries of that expert -- goes to route_rel.
+// After the kernel route_counts holds the per-expert histogram; the consumer
+// adds the exclusive prefix of the counts to place rows.  Rows of one expert
+// are grouped by tile in the order the tiles reserved them; that order does
+// not change any output, since every GEMM row depends only on its own input.
+__device__ void route_tile(const KParams& p, int tile, int BT, const int* sIdx, int* s_base) {
+  const int nt = BT * p.k;
+  const long long e0 = (long long)tile * nt;
+  const long long n = (long long)p.T * p.k;
+  const int live = (int)((n - e0) < nt ? (n - e0) : nt);
+  for (int e = threadIdx.x; e < p.E; e += SL_THREADS) {
+    int c = 0;
+    for (int j = 0; j < live; ++j) c += (sIdx[j] == e) ? 1 : 0;
+    s_base[e] = c ? atomicAdd(&p.route_counts[e], c) : 0;
+  }
+  __syncthreads();
+  for (int i = threadIdx.x; i < live; i += SL_THREADS) {
+    const int e = sIdx[i];
+    int rank = 0;
+    for (int j = 0; j < i; ++j) rank += (sIdx[j] == e) ? 1 : 0;
+    p.route_rel[e0 + i] = s_base[e] + rank;
+  }
+  __syncthreads();
+}
+
 template <typename TX, int XC, int TPT, int NB>
 __global__ void __launch_bounds__(SL_THREADS) gate_slices_kernel(const KParams p, int S) {
   extern __shared__ float smem_f[];
@@ -391,9 +426,12 @@ __global__ void __launch_bounds__(SL_THREADS) gate_slices_kernel(const KParams p
   float* sW = smem_f;                   // [O][d]
   float* sRed = sW + (size_t)O * p.d;   // [NB][RS]
   float* sLog = sRed + NB * RS;         // [BT][O]
+  int* sIdx = reinterpret_cast<int*>(sLog + BT * O);  // [BT * k] this tile's expert ids
+  __shared__ int s_base[128];
   const int jq = threadIdx.x % JQ;
   const int sl = threadIdx.x / JQ;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_trigger();
 
   {  // stage the gate rows, eight 16-byte loads in flight per thread
     const int n4 = O * p.d / 4;
@@ -415,6 +453,7 @@ __global__ void __launch_bounds__(SL_THREADS) gate_slices_kernel(const KParams p
       }
     }
   }
+  pdl_wait();
   __syncthreads();
 
   const TX* X = reinterpret_cast<const TX*>(p.X);
@@ -476,15 +515,17 @@ __global__ void __launch_bounds__(SL_THREADS) gate_slices_kernel(const KParams p
     }
     for (int jj = warp; jj < BT; jj += SL_THREADS / 32) {
       const int tok = tile * BT + jj;
-      if (tok < p.T) decide_token_warp(p, sLog + jj * O, tok, lane);
+      if (tok < p.T) decide_token_warp(p, sLog + jj * O, tok, lane, p.route_counts ? sIdx + jj * p.k : nullptr);
     }
     __syncthreads();
+    if (p.route_counts) route_tile(p, tile, BT, sIdx, s_base);
   }
 }
 
 }  // namespace
 
-cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
+cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed) {
+  if (routed) *routed = false;
   KParams p;
   p.X = a.X;
   p.W_local = a.W_local;
@@ -500,6 +541,8 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
   p.renorm = a.renorm;
   p.topk_idx = a.topk_idx;
   p.topk_w = a.topk_w;
+  p.route_counts = nullptr;
+  p.route_rel = nullptr;
   const int O = a.E + (a.K == 1 ? 0 : a.K);
   cudaError_t e;
   // Slice kernel when every gate row fits in shared memory next to the
@@ -517,9 +560,17 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
     }
     const int NB = O <= 16 ? 16 : 32;
     const int BT = S ? (SL_THREADS / S) * TPT : 0;
-    const size_t smem = (size_t)O * a.d * 4 + (size_t)NB * (S * BT + SL_RED_PAD) * 4 + (size_t)BT * O * 4;
+    const size_t smem = (size_t)O * a.d * 4 + (size_t)NB * (S * BT + SL_RED_PAD) * 4 + (size_t)BT * O * 4 +
+                        (size_t)BT * a.k * 4;
     if (S && smem <= 160 * 1024) {
       const long long tiles = (a.T + BT - 1) / BT;
+      if (a.route_counts && a.route_rel) {
+        p.route_counts = a.route_counts;
+        p.route_rel = a.route_rel;
+        e = cudaMemsetAsync(a.route_counts, 0, sizeof(int32_t) * a.E, s);
+        if (e != cudaSuccess) return e;
+        if (routed) *routed = true;
+      }
       const int per_sm = smem <= 72 * 1024 ? 3 : (smem <= 110 * 1024 ? 2 : 1);
       long long blocks = tiles < (long long)sm_count() * per_sm ? tiles : (long long)sm_count() * per_sm;
       if (blocks < 1) blocks = 1;
@@ -529,7 +580,8 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
   do {                                                                                                      \
     e = ensure_smem_attr(reinterpret_cast<const void*>(gate_slices_kernel<TX, XC, TP, NBV>), (int)smem);     \
     if (e != cudaSuccess) return e;                                                                         \
-    gate_slices_kernel<TX, XC, TP, NBV><<<(int)blocks, SL_THREADS, smem, s>>>(p, S);                        \
+    e = launch_kernel(gate_slices_kernel<TX, XC, TP, NBV>, dim3((int)blocks), dim3(SL_THREADS), smem, s, p, S); \
+    if (e != cudaSuccess) return e;                                                                         \
   } while (0)
 #define EC2MOE_SLICES_NB(TX, XC, TP) \
   do {                               \
@@ -565,7 +617,8 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s) {
   do {                                                                                                      \
     e = ensure_smem_attr(reinterpret_cast<const void*>(gate_topk_kernel<TX, WS>), (int)smem);            \
     if (e != cudaSuccess) return e;                                                                         \
-    gate_topk_kernel<TX, WS><<<blocks, WARPS * 32, smem, s>>>(p);                                           \
+    e = launch_kernel(gate_topk_kernel<TX, WS>, dim3(blocks), dim3(WARPS * 32), smem, s, p);                 \
+    if (e != cudaSuccess) return e;                                                                         \
   } while (0)
   if (bf16) {
     if (w_smem) EC2MOE_GATE_LAUNCH(__nv_bfloat16, true); else EC2MOE_GATE_LAUNCH(__nv_bfloat16, false);

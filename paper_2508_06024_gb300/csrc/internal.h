@@ -29,6 +29,30 @@ class KernelScope {
 
 int sm_count();
 
+// Whether the next launch of the current public call may overlap its
+// predecessor (programmatic dependent launch): every launch but the first of
+// a call, unless EC2MOE_NO_PDL=1 is set in the environment.  The first launch
+// keeps full stream ordering, so work the caller enqueued earlier is never
+// raced.  Kernels only read data produced earlier in the stream after
+// griddepcontrol.wait.
+bool next_launch_pdl();
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                                 Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = next_launch_pdl() ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // cudaFuncSetAttribute(MaxDynamicSharedMemorySize) once per (device, kernel),
 // raised only when a launch needs more than was set before.
 cudaError_t ensure_smem_attr(const void* kernel, int bytes);
@@ -44,8 +68,22 @@ struct GateArgs {
   int T, d, E, K, k, renorm;
   int32_t* topk_idx;
   float* topk_w;
+  // Routing fused into the gate (layer path; both nullptr: gate only): the
+  // kernel fills route_counts (the per-expert histogram; cleared by the host
+  // first) and route_rel[T*k] (each entry's row relative to its expert's
+  // first row).  Consumers place rows at offsets[e] + route_rel[i].
+  int32_t* route_counts;
+  int32_t* route_rel;
 };
-cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s);
+// Launches the gate; with the routing fields set, also fills them when the
+// fused path applies (*routed = true), else gate only.
+cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed = nullptr);
+// Rows into expert order from relative positions: for entry i (token i / k),
+// pos = offsets[e] + rel[i] with offsets = exclusive prefix of counts;
+// dst[pos] = src[i / k], perm[pos] = i; block 0 writes offsets[0..E].
+cudaError_t launch_gather_rel(const void* src, void* dst, const int32_t* topk_idx, const int32_t* counts,
+                              const int32_t* rel, int32_t* perm, int32_t* offsets, int E, long long n, int k,
+                              int width, bool bf16, cudaStream_t s);
 
 // ----------------------------------------------------------- routing tables / moves
 int route_blocks(long long n_entries);  // per-block histogram blocks
@@ -66,7 +104,7 @@ cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, v
                            bool bf16, cudaStream_t s);
 
 // ------------------------------------------------------------------ grouped GEMMs
-enum Epi { EPI_STORE = 0, EPI_GELU = 1, EPI_SWIGLU = 2, EPI_SCATTER = 3 };
+enum Epi { EPI_STORE = 0, EPI_GELU = 1, EPI_SWIGLU = 2, EPI_SCATTER = 3, EPI_REPLICATE = 4 };
 
 // Group g of a grouped GEMM owns rows [row0(g), row0(g) + M_g) of A and of the
 // pre-scatter output, with
@@ -82,8 +120,22 @@ struct GemmArgs {
   int N, K, b_group_rows;
   void* out; long long ldo;          // output pitch in elements
   const int32_t* perm;               // EPI_SCATTER: dest row = perm[out_row]
+                                     // EPI_REPLICATE: dest rows perm[out_row*rep_k + s], s < rep_k
   const float* scale;                // EPI_SCATTER: multiply by scale[dest] (nullptr = 1)
+  int rep_k;                         // EPI_REPLICATE: copies per row
+  long long self_row_base;           // EPI_REPLICATE: also write row self_row_base + out_row (< 0: no)
+  // EPI_REPLICATE with relative positions (rep_counts != nullptr): `perm`
+  // holds rows relative to each expert's first row; the destination of entry
+  // i is offsets[e] + perm[i] with e = rep_idx[i] and offsets the exclusive
+  // prefix of rep_counts[0..rep_E); the epilogue also writes rep_perm_out[dest]
+  // = i, and CTA 0 writes rep_offsets_out[0..rep_E].
+  const int32_t* rep_counts;
+  const int32_t* rep_idx;
+  int32_t* rep_perm_out;
+  int32_t* rep_offsets_out;
+  int rep_E;
   long long max_rows;                // upper bound of sum_g M_g (for the grid size)
+  int g_active;                      // groups expected to hold rows (tile-count estimate; 0 = G)
   long long timeout_cycles;          // bounded-wait budget (tensor-core path)
   const char* name;                  // label for per-launch profiling (nullptr = by epilogue)
 };

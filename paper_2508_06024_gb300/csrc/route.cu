@@ -16,7 +16,7 @@
 
 #include <mutex>
 
-#include "../../include/ec2moe.h"
+#include "ec2moe.h"
 #include "common.cuh"
 #include "internal.h"
 
@@ -36,6 +36,8 @@ constexpr int MAXE = 128;
 
 __global__ void __launch_bounds__(CHUNK) route_count_kernel(const int32_t* __restrict__ idx, long long n, int E,
                                                             int32_t* __restrict__ blk_counts) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ int hist[MAXE];
   for (int e = threadIdx.x; e < E; e += blockDim.x) hist[e] = 0;
   __syncthreads();
@@ -49,6 +51,8 @@ __global__ void __launch_bounds__(CHUNK) route_scatter_kernel(const int32_t* __r
                                                               const int32_t* __restrict__ blk_counts, int nblk,
                                                               int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
                                                               int32_t* __restrict__ perm, int32_t* __restrict__ inv_perm) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ int s_pre[MAXE];           // entries of expert e in earlier blocks
   __shared__ int s_base[MAXE];          // offsets[e] + s_pre[e]
   __shared__ int s_tot[MAXE];
@@ -107,9 +111,86 @@ __global__ void __launch_bounds__(CHUNK) route_scatter_kernel(const int32_t* __r
   }
 }
 
+// Whole routing in one block for up to SMALL_MAX entries: histogram
+// (warp-aggregated shared atomics), exclusive scan, then the entries in
+// 1024-entry rounds in order, each ranked inside the round (warp match +
+// prefix over warps) on top of per-expert running bases.  Same results as the
+// two-kernel path.
+constexpr int SMALL_MAX = 16384;
+
+__global__ void __launch_bounds__(CHUNK) route_small_kernel(const int32_t* __restrict__ idx, int n, int E,
+                                                            int32_t* __restrict__ counts, int32_t* __restrict__ offsets,
+                                                            int32_t* __restrict__ perm, int32_t* __restrict__ inv_perm) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ int hist[MAXE];
+  __shared__ int base[MAXE];
+  __shared__ int tot[MAXE];
+  __shared__ int wcnt[CHUNK / 32][MAXE];
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  for (int e = threadIdx.x; e < E; e += blockDim.x) hist[e] = 0;
+  __syncthreads();
+  for (int i0 = 0; i0 < n; i0 += CHUNK) {
+    const int i = i0 + threadIdx.x;
+    const bool live = i < n;
+    const unsigned act = __ballot_sync(0xffffffffu, live);
+    if (live) {
+      const int e = idx[i];
+      const unsigned same = __match_any_sync(act, e);
+      if ((same & ((1u << lane) - 1u)) == 0) atomicAdd(&hist[e], __popc(same));
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int e = 0; e < E; ++e) {
+      base[e] = acc;
+      counts[e] = hist[e];
+      offsets[e] = acc;
+      acc += hist[e];
+    }
+    offsets[E] = acc;
+  }
+  for (int i0 = 0; i0 < n; i0 += CHUNK) {
+    for (int c = threadIdx.x; c < (CHUNK / 32) * MAXE; c += blockDim.x) (&wcnt[0][0])[c] = 0;
+    __syncthreads();
+    const int i = i0 + threadIdx.x;
+    const bool live = i < n;
+    const unsigned act = __ballot_sync(0xffffffffu, live);
+    int e = 0, rank_w = 0;
+    if (live) {
+      e = idx[i];
+      const unsigned same = __match_any_sync(act, e);
+      rank_w = __popc(same & ((1u << lane) - 1u));
+      if (rank_w == 0) wcnt[warp][e] = __popc(same);
+    }
+    __syncthreads();
+    for (int ee = threadIdx.x; ee < E; ee += blockDim.x) {
+      int acc = 0;
+      for (int w = 0; w < CHUNK / 32; ++w) {
+        const int c = wcnt[w][ee];
+        wcnt[w][ee] = acc;
+        acc += c;
+      }
+      tot[ee] = acc;
+    }
+    __syncthreads();
+    if (live) {
+      const int pos = base[e] + wcnt[warp][e] + rank_w;
+      perm[pos] = i;
+      if (inv_perm) inv_perm[i] = pos;
+    }
+    __syncthreads();
+    for (int ee = threadIdx.x; ee < E; ee += blockDim.x) base[ee] += tot[ee];
+  }
+}
+
 // dst[p] = src[perm[p] / k]; one warp per row, 16-byte lanes.
 __global__ void gather_rows_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
                                    const int32_t* __restrict__ perm, long long rows, int k, int row_bytes) {
+  pdl_trigger();
+  pdl_wait();
   const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
   for (long long r = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += warps) {
@@ -120,10 +201,44 @@ __global__ void gather_rows_kernel(const uint8_t* __restrict__ src, uint8_t* __r
   }
 }
 
+// Rows into expert order from relative positions (routing fused into the
+// gate): pos = offsets[e] + rel[i], dst[pos] = src[i / k], perm[pos] = i.
+// Each block derives the offsets from the counts; block 0 publishes them.
+__global__ void gather_rel_kernel(const uint8_t* __restrict__ src, uint8_t* __restrict__ dst,
+                                  const int32_t* __restrict__ idx, const int32_t* __restrict__ counts,
+                                  const int32_t* __restrict__ rel, int32_t* __restrict__ perm,
+                                  int32_t* __restrict__ offsets, int E, long long n, int k, int row_bytes) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ int s_off[MAXE + 1];
+  if (threadIdx.x == 0) {
+    int run = 0;
+    for (int e = 0; e < E; ++e) {
+      s_off[e] = run;
+      run += counts[e];
+    }
+    s_off[E] = run;
+    if (blockIdx.x == 0)
+      for (int e = 0; e <= E; ++e) offsets[e] = s_off[e];
+  }
+  __syncthreads();
+  const int lane = threadIdx.x & 31;
+  const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
+  for (long long i = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < n; i += warps) {
+    const int pos = s_off[idx[i]] + rel[i];
+    if (lane == 0) perm[pos] = static_cast<int32_t>(i);
+    const U4* sr = reinterpret_cast<const U4*>(src + (i / k) * row_bytes);
+    U4* dr = reinterpret_cast<U4*>(dst + (long long)pos * row_bytes);
+    for (int c = lane; c < row_bytes / 16; c += 32) dr[c] = sr[c];
+  }
+}
+
 // y[t] = sum_s slot[t*k+s] + sum_j shared[j*T+t] in that order, fp32 sum.
 template <typename TE>
 __global__ void combine_kernel(const TE* __restrict__ slot, const TE* __restrict__ shared, int n_shared,
                                TE* __restrict__ Y, int T, int k, int d) {
+  pdl_trigger();
+  pdl_wait();
   const int per_row = d / 8;
   const long long total = (long long)T * per_row;
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
@@ -159,13 +274,21 @@ cudaError_t launch_route(const int32_t* topk_idx, long long n, int E, int32_t* b
     if (e != cudaSuccess) return e;
     return cudaMemsetAsync(offsets, 0, sizeof(int32_t) * (E + 1), s);
   }
+  if (n <= SMALL_MAX) {
+    KernelScope ks("route", s);
+    return launch_kernel(route_small_kernel, dim3(1), dim3(CHUNK), 0, s, topk_idx, static_cast<int>(n), E, counts,
+                         offsets, perm, inv_perm);
+  }
   {
     KernelScope ks("route_count", s);
-    route_count_kernel<<<nblk, CHUNK, 0, s>>>(topk_idx, n, E, blk_counts);
+    cudaError_t e = launch_kernel(route_count_kernel, dim3(nblk), dim3(CHUNK), 0, s, topk_idx, n, E, blk_counts);
+    if (e != cudaSuccess) return e;
   }
   {
     KernelScope ks("route_scatter", s);
-    route_scatter_kernel<<<nblk, CHUNK, 0, s>>>(topk_idx, n, E, blk_counts, nblk, counts, offsets, perm, inv_perm);
+    cudaError_t e = launch_kernel(route_scatter_kernel, dim3(nblk), dim3(CHUNK), 0, s, topk_idx, n, E,
+                                  (const int32_t*)blk_counts, nblk, counts, offsets, perm, inv_perm);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }
@@ -211,10 +334,26 @@ cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long 
   if (blocks > cap) blocks = cap;
   {
     KernelScope ks("gather_rows", s);
-    gather_rows_kernel<<<static_cast<int>(blocks), warps_per_block * 32, 0, s>>>(
-        static_cast<const uint8_t*>(src), static_cast<uint8_t*>(dst), perm, rows, k, row_bytes);
+    cudaError_t e = launch_kernel(gather_rows_kernel, dim3(static_cast<int>(blocks)), dim3(warps_per_block * 32), 0, s,
+                                  static_cast<const uint8_t*>(src), static_cast<uint8_t*>(dst), perm, rows, k, row_bytes);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
+}
+
+cudaError_t launch_gather_rel(const void* src, void* dst, const int32_t* topk_idx, const int32_t* counts,
+                              const int32_t* rel, int32_t* perm, int32_t* offsets, int E, long long n, int k,
+                              int width, bool bf16, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const int row_bytes = width * (bf16 ? 2 : 4);
+  const int warps_per_block = 8;
+  long long blocks = (n + warps_per_block - 1) / warps_per_block;
+  const long long cap = (long long)sm_count() * 8;
+  if (blocks > cap) blocks = cap;
+  KernelScope ks("gather_rows", s);
+  return launch_kernel(gather_rel_kernel, dim3(static_cast<int>(blocks)), dim3(warps_per_block * 32), 0, s,
+                       static_cast<const uint8_t*>(src), static_cast<uint8_t*>(dst), topk_idx, counts, rel, perm,
+                       offsets, E, n, k, row_bytes);
 }
 
 cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d, bool bf16,
@@ -226,13 +365,15 @@ cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, v
   if (blocks > cap) blocks = cap;
   KernelScope ks("combine", s);
   if (bf16) {
-    combine_kernel<__nv_bfloat16><<<static_cast<int>(blocks), 256, 0, s>>>(
-        static_cast<const __nv_bfloat16*>(slot), static_cast<const __nv_bfloat16*>(shared), shared ? n_shared : 0,
-        static_cast<__nv_bfloat16*>(Y), T, k, d);
+    cudaError_t e = launch_kernel(combine_kernel<__nv_bfloat16>, dim3(static_cast<int>(blocks)), dim3(256), 0, s,
+                                  static_cast<const __nv_bfloat16*>(slot), static_cast<const __nv_bfloat16*>(shared),
+                                  shared ? n_shared : 0, static_cast<__nv_bfloat16*>(Y), T, k, d);
+    if (e != cudaSuccess) return e;
   } else {
-    combine_kernel<float><<<static_cast<int>(blocks), 256, 0, s>>>(static_cast<const float*>(slot),
-                                                                   static_cast<const float*>(shared),
-                                                                   shared ? n_shared : 0, static_cast<float*>(Y), T, k, d);
+    cudaError_t e = launch_kernel(combine_kernel<float>, dim3(static_cast<int>(blocks)), dim3(256), 0, s,
+                                  static_cast<const float*>(slot), static_cast<const float*>(shared),
+                                  shared ? n_shared : 0, static_cast<float*>(Y), T, k, d);
+    if (e != cudaSuccess) return e;
   }
   return cudaGetLastError();
 }

@@ -31,12 +31,16 @@ struct SParams {
   long long ldo;
   const int32_t* perm;
   const float* scale;
+  int rep_k;
+  long long self_row_base;
   int n_tiles_n;
   long long a_rows, b_rows;
 };
 
 template <int EPI>
 __global__ void __launch_bounds__(256) simt_gemm_kernel(const SParams p) {
+  pdl_trigger();
+  pdl_wait();
   __shared__ int tile_prefix[MAX_GROUPS + 1];
   __shared__ int row0[MAX_GROUPS];
   __shared__ float sA[TK][TM + 4];
@@ -123,7 +127,12 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SParams p) {
         if (EPI == EPI_GELU) v = gelu_erf(v);
         if (EPI == EPI_SWIGLU) v = silu(v) * acc2[i][j];
         if (EPI == EPI_SCATTER) v *= sc;
-        p.out[dest * p.ldo + col] = v;
+        if (EPI == EPI_REPLICATE) {
+          for (int r = 0; r < p.rep_k; ++r) p.out[(long long)p.perm[out_row * p.rep_k + r] * p.ldo + col] = v;
+          if (p.self_row_base >= 0) p.out[(p.self_row_base + out_row) * p.ldo + col] = v;
+        } else {
+          p.out[dest * p.ldo + col] = v;
+        }
       }
     }
   }
@@ -150,6 +159,8 @@ cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s) {
   p.ldo = a.ldo;
   p.perm = a.perm;
   p.scale = a.scale;
+  p.rep_k = a.rep_k;
+  p.self_row_base = a.self_row_base;
   p.n_tiles_n = (a.N + TN - 1) / TN;
   p.a_rows = a.a_rows;
   p.b_rows = a.b_rows;
@@ -157,13 +168,16 @@ cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s) {
   const long long cap = (long long)sm_count() * 8;
   const int grid = static_cast<int>(tiles < cap ? (tiles > 0 ? tiles : 1) : cap);
   KernelScope ks(a.name ? a.name : "gemm_simt", s);
+  cudaError_t e = cudaSuccess;
   switch (epi) {
-    case EPI_STORE: simt_gemm_kernel<EPI_STORE><<<grid, 256, 0, s>>>(p); break;
-    case EPI_GELU: simt_gemm_kernel<EPI_GELU><<<grid, 256, 0, s>>>(p); break;
-    case EPI_SWIGLU: simt_gemm_kernel<EPI_SWIGLU><<<grid, 256, 0, s>>>(p); break;
-    case EPI_SCATTER: simt_gemm_kernel<EPI_SCATTER><<<grid, 256, 0, s>>>(p); break;
+    case EPI_STORE: e = launch_kernel(simt_gemm_kernel<EPI_STORE>, dim3(grid), dim3(256), 0, s, p); break;
+    case EPI_GELU: e = launch_kernel(simt_gemm_kernel<EPI_GELU>, dim3(grid), dim3(256), 0, s, p); break;
+    case EPI_SWIGLU: e = launch_kernel(simt_gemm_kernel<EPI_SWIGLU>, dim3(grid), dim3(256), 0, s, p); break;
+    case EPI_SCATTER: e = launch_kernel(simt_gemm_kernel<EPI_SCATTER>, dim3(grid), dim3(256), 0, s, p); break;
+    case EPI_REPLICATE: e = launch_kernel(simt_gemm_kernel<EPI_REPLICATE>, dim3(grid), dim3(256), 0, s, p); break;
     default: return cudaErrorInvalidValue;
   }
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -55,6 +55,13 @@ struct Params {
   long long ldo;
   const int32_t* perm;
   const float* scale;
+  int rep_k;
+  long long self_row_base;
+  const int32_t* rep_counts;
+  const int32_t* rep_idx;
+  int32_t* rep_perm_out;
+  int32_t* rep_offsets_out;
+  int rep_E;
   long long timeout;
   int n_tiles_n;
 };
@@ -187,6 +194,33 @@ __device__ __forceinline__ void tmem_ld(uint32_t taddr, float* v) {
   else tmem_ld16(taddr, v);
 }
 
+// Issue-only TMEM loads (the caller waits with tmem_wait once for several).
+__device__ __forceinline__ void tmem_ld32_nw(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld16_nw(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+}
+template <int CW>
+__device__ __forceinline__ void tmem_ld_nw(uint32_t taddr, uint32_t* r) {
+  if (CW == 32) tmem_ld32_nw(taddr, r);
+  else tmem_ld16_nw(taddr, r);
+}
+__device__ __forceinline__ void tmem_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
 // ------------------------------------------------------------------ tile schedule
 struct TileCoord {
   int g, m_blk, n_blk;
@@ -214,7 +248,11 @@ struct Cfg {
   static_assert(HALF % CW == 0 && CW % 16 == 0, "epilogue chunks must tile each half exactly");
   static constexpr int TMEM_COLS = pow2_at_least(2 * BN);  // two accumulators
   static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8;
-  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES + 16 + 2 * (MAX_GROUPS + 1) * 4;
+  static constexpr int STG_PITCH = CW * 2 + 16;          // bytes per staged row (padded: conflict-free)
+  static constexpr int STG_BYTES = EPI_WARPS * 32 * STG_PITCH;
+  static constexpr int OFF_INTS = 132;  // expert offsets of EPI_REPLICATE's relative mode (<= 128 + 1, padded)
+  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES + 16 + 2 * (MAX_GROUPS + 1) * 4 + OFF_INTS * 4 +
+                              STG_BYTES;
 };
 
 template <int BN, int EPI, int STAGES>
@@ -236,9 +274,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   int* tile_prefix = reinterpret_cast<int*>(tmem_slot + 4);
   int* row0 = tile_prefix + (MAX_GROUPS + 1);
+  int* s_off = row0 + MAX_GROUPS + 1;                                    // [C::OFF_INTS]
+  uint8_t* stg_all = reinterpret_cast<uint8_t*>(s_off + C::OFF_INTS);  // epilogue staging, 16-byte aligned
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  // Barrier set-up, TMEM allocation and descriptor prefetch overlap the
+  // previous kernel; everything that reads its results comes after pdl_wait.
+  pdl_trigger();
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -253,6 +296,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    pdl_wait();
     // Per-group tile prefix (m tiles) and first rows.
     int acc = 0;
     tile_prefix[0] = 0;
@@ -269,6 +313,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       acc += (mg + BM - 1) / BM;
       tile_prefix[g + 1] = acc;
     }
+    if (EPI == EPI_REPLICATE && p.rep_counts) {
+      int run = 0;
+      for (int e = 0; e < p.rep_E; ++e) {
+        s_off[e] = run;
+        run += p.rep_counts[e];
+      }
+      s_off[p.rep_E] = run;
+      if (blockIdx.x == 0)
+        for (int e = 0; e <= p.rep_E; ++e) p.rep_offsets_out[e] = s_off[e];
+    }
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
@@ -284,6 +338,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_wait();
   const uint32_t tmem_base = *tmem_slot;
   const int n_tiles = tile_prefix[p.G] * p.n_tiles_n;
   const int num_kb = (p.K + BK - 1) / BK;
@@ -402,28 +457,91 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         dest = p.perm ? p.perm[out_row] : out_row;
         if (p.scale) sc = p.scale[dest];
       }
+      // EPI_REPLICATE: this row's destinations, read once per tile.
+      int rdst[8];
+      if (EPI == EPI_REPLICATE) {
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+          rdst[r] = 0;
+          if (valid && r < p.rep_k) {
+            const long long entry = out_row * p.rep_k + r;
+            int dst = p.perm[entry];
+            if (p.rep_counts) {
+              dst += s_off[p.rep_idx[entry]];
+              p.rep_perm_out[dst] = static_cast<int32_t>(entry);
+            }
+            rdst[r] = dst;
+          }
+        }
+      }
       const uint32_t t_row = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
-      __nv_bfloat16* orow = reinterpret_cast<__nv_bfloat16*>(p.out) + dest * p.ldo;
+      // Each chunk of 32 rows x CW columns is staged in shared memory (thread =
+      // row) and written back with 4 lanes per row segment, so a warp store
+      // covers CW*2/16 ... contiguous 16-byte pieces of 32/(CW/8) rows.
+      uint8_t* stg = stg_all + (warp - 2) * 32 * C::STG_PITCH;
+      constexpr int SEGS = C::CW / 8;           // 16-byte segments per row
+      constexpr int ROWS_PER_PASS = 32 / SEGS;  // rows a warp store covers
+      // Two chunks' TMEM loads are issued before one wait (half as many waits);
+      // a half with an odd number of chunks ends on a single chunk.
+      constexpr int NCH = C::HALF / C::CW;
+      uint32_t rv[2][C::CW], ru[2][C::CW];
 #pragma unroll 1
-      for (int c0 = half * C::HALF; c0 < (half + 1) * C::HALF; c0 += C::CW) {
+      for (int ci = 0; ci < NCH; ++ci) {
+        const int c0 = half * C::HALF + ci * C::CW;
+        const int slot = ci & 1;
+        if (slot == 0) {
+          tmem_ld_nw<C::CW>(t_row + c0, rv[0]);
+          if (EPI == EPI_SWIGLU) tmem_ld_nw<C::CW>(t_row + c0 + BN / 2, ru[0]);
+          if (ci + 1 < NCH) {
+            tmem_ld_nw<C::CW>(t_row + c0 + C::CW, rv[1]);
+            if (EPI == EPI_SWIGLU) tmem_ld_nw<C::CW>(t_row + c0 + C::CW + BN / 2, ru[1]);
+          }
+          tmem_wait();
+        }
         const int col = tc.n_blk * C::BN_OUT + c0;
         float v[C::CW];
-        tmem_ld<C::CW>(t_row + c0, v);
-        if (EPI == EPI_SWIGLU) {
-          float u[C::CW];
-          tmem_ld<C::CW>(t_row + c0 + BN / 2, u);
 #pragma unroll
-          for (int i = 0; i < C::CW; ++i) v[i] = silu(v[i]) * u[i];
+        for (int i = 0; i < C::CW; ++i) v[i] = __uint_as_float(slot ? rv[1][i] : rv[0][i]);
+        if (EPI == EPI_SWIGLU) {
+#pragma unroll
+          for (int i = 0; i < C::CW; ++i) v[i] = silu_bf16out(v[i]) * __uint_as_float(slot ? ru[1][i] : ru[0][i]);
         } else if (EPI == EPI_GELU) {
 #pragma unroll
-          for (int i = 0; i < C::CW; ++i) v[i] = gelu_erf(v[i]);
+          for (int i = 0; i < C::CW; ++i) v[i] = gelu_bf16out(v[i]);
         } else if (EPI == EPI_SCATTER) {
 #pragma unroll
           for (int i = 0; i < C::CW; ++i) v[i] *= sc;
         }
-        if (valid && col < p.N) {
+        if (col >= p.N) continue;  // uniform across the warp
+        __syncwarp();
 #pragma unroll
-          for (int j = 0; j < C::CW / 8; ++j) store8(orow + col + 8 * j, v + 8 * j);
+        for (int j = 0; j < SEGS; ++j) {
+          U4 q4{pack_bf16x2(v[8 * j + 0], v[8 * j + 1]), pack_bf16x2(v[8 * j + 2], v[8 * j + 3]),
+                pack_bf16x2(v[8 * j + 4], v[8 * j + 5]), pack_bf16x2(v[8 * j + 6], v[8 * j + 7])};
+          *reinterpret_cast<U4*>(stg + lane * C::STG_PITCH + 16 * j) = q4;
+        }
+        __syncwarp();
+        const int sg = lane % SEGS;
+#pragma unroll
+        for (int pass = 0; pass < SEGS; ++pass) {
+          const int rr = pass * ROWS_PER_PASS + lane / SEGS;  // staged row this lane writes
+          const bool rvalid = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr) != 0;
+          const U4 q4 = *reinterpret_cast<const U4*>(stg + rr * C::STG_PITCH + 16 * sg);
+          if (EPI == EPI_REPLICATE) {
+            const long long orow_r = __shfl_sync(0xffffffffu, out_row, rr);
+            __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(p.out);
+#pragma unroll
+            for (int r = 0; r < 8; ++r) {
+              const int dr = __shfl_sync(0xffffffffu, rdst[r], rr);
+              if (rvalid && r < p.rep_k) *reinterpret_cast<U4*>(ob + (long long)dr * p.ldo + col + 8 * sg) = q4;
+            }
+            if (rvalid && p.self_row_base >= 0)
+              *reinterpret_cast<U4*>(ob + (p.self_row_base + orow_r) * p.ldo + col + 8 * sg) = q4;
+          } else {
+            const long long drow = __shfl_sync(0xffffffffu, dest, rr);
+            if (rvalid)
+              *reinterpret_cast<U4*>(reinterpret_cast<__nv_bfloat16*>(p.out) + drow * p.ldo + col + 8 * sg) = q4;
+          }
         }
       }
       tc_fence_before();
@@ -518,6 +636,7 @@ const char* kernel_name(int epi) {
     case EPI_GELU: return "gemm_tc_gelu";
     case EPI_SWIGLU: return "gemm_tc_swiglu";
     case EPI_SCATTER: return "gemm_tc_scatter";
+    case EPI_REPLICATE: return "gemm_tc_replicate";
     default: return "gemm_tc_store";
   }
 }
@@ -550,6 +669,13 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   p.ldo = a.ldo;
   p.perm = a.perm;
   p.scale = a.scale;
+  p.rep_k = a.rep_k;
+  p.self_row_base = a.self_row_base;
+  p.rep_counts = a.rep_counts;
+  p.rep_idx = a.rep_idx;
+  p.rep_perm_out = a.rep_perm_out;
+  p.rep_offsets_out = a.rep_offsets_out;
+  p.rep_E = a.rep_E;
   p.timeout = a.timeout_cycles;
   p.n_tiles_n = (a.N + C::BN_OUT - 1) / C::BN_OUT;
   const long long m_tiles_max = a.max_rows / BM + a.G;
@@ -557,7 +683,9 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
   if (grid < 1) grid = 1;
   KernelScope ks(a.name ? a.name : kernel_name(EPI), s);
-  tc_gemm_kernel<BN, EPI, STAGES><<<grid, NUM_THREADS, C::SMEM, s>>>(mA, mB, mB2, p);
+  cudaError_t le = launch_kernel(tc_gemm_kernel<BN, EPI, STAGES>, dim3(grid), dim3(NUM_THREADS), (size_t)C::SMEM, s, mA,
+                                 mB, mB2, p);
+  if (le != cudaSuccess) return le;
   return cudaGetLastError();
 }
 
@@ -578,22 +706,33 @@ cudaError_t launch_epi(const GemmArgs& a, int bn, cudaStream_t s) {
   return cudaErrorInvalidValue;
 }
 
-// N-tile choice: the widest tile whose expected tile count still gives every
-// SM work (>= 90% of the SMs), else the narrowest (most parallel) tile.  The
-// m-tile count of a grouped GEMM is only known on the device; half a partial
-// tile per group is expected.
+// N-tile choice.  Each candidate is scored by its wave efficiency (tiles over
+// whole waves of one tile per SM) times a per-tile efficiency that falls with
+// the tile width (narrow tiles move more operand bytes per FLOP).  The m-tile
+// count of a grouped GEMM is only known on the device; half a partial tile
+// per group is expected.
 int choose_bn(const GemmArgs& a, int epi) {
-  const double m_tiles = (double)a.max_rows / BM + (a.G > 1 ? 0.5 * a.G : 0.0) + (a.G == 1 && a.max_rows % BM ? 1 : 0);
+  const int ga = a.g_active > 0 ? a.g_active : a.G;
+  const double m_tiles = (double)a.max_rows / BM + (a.G > 1 ? 0.5 * ga : 0.0) + (a.G == 1 && a.max_rows % BM ? 1 : 0);
   const int sms = sm_count();
   const int cands[5] = {256, 192, 128, 64, 32};
+  const double tile_eff[5] = {1.0, 0.97, 0.9, 0.75, 0.6};
   int pick = 0;
-  for (int bn : cands) {
+  double best = -1.0;
+  for (int i = 0; i < 5; ++i) {
+    const int bn = cands[i];
     const int out = (epi == EPI_SWIGLU) ? bn / 2 : bn;
     if (epi == EPI_SWIGLU && bn < 64) continue;
-    if (out > a.N && bn != 32 && !(epi == EPI_SWIGLU && bn == 64)) continue;  // no wider than N
-    pick = bn;
+    if (out > a.N && !(out == 32 || (epi == EPI_SWIGLU && bn == 64))) continue;  // no wider than N
     const double tiles = m_tiles * ((a.N + out - 1) / out);
-    if (tiles >= 0.9 * sms) return bn;
+    const double waves = tiles / sms;
+    const double wave_eff = tiles / (sms * (waves <= 1.0 ? 1.0 : static_cast<double>((long long)(waves + 0.999))));
+    const double useful = (double)a.N / (((a.N + out - 1) / out) * out);  // columns wasted on a partial N tile
+    const double score = wave_eff * tile_eff[i] * useful;
+    if (score > best + 1e-9) {
+      best = score;
+      pick = bn;
+    }
   }
   return pick;
 }
@@ -608,6 +747,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
     case EPI_GELU: return launch_epi<EPI_GELU>(a, bn, s);
     case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, s);
     case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, s);
+    case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, s);
   }
   return cudaErrorInvalidValue;
 }
