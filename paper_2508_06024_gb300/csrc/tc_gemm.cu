@@ -9,12 +9,12 @@
 // step-specific op (plain store, GELU, SwiGLU, or gate-scale + scatter to the
 // token's slot for the combine of Eq. 1).
 //
-// CTA layout (320 threads):
+// CTA layout (576 threads):
 //   warp 0      TMA producer (one elected lane)
 //   warp 1      TMEM allocator + MMA issuer (one elected lane)
-//   warps 2..9  epilogue: TMEM -> registers -> global.  Warp w may only read
-//               TMEM lanes 32*(w%4) .. +31 (rows of the 128-row tile); the two
-//               warps of a lane quadrant split the tile's columns in halves.
+//   warps 2..17 epilogue: TMEM -> registers -> global.  Warp w may only read
+//               TMEM lanes 32*(w%4) .. +31 (rows of the 128-row tile); the
+//               four warps of a lane quadrant split the tile's columns.
 // Pipelines: STAGES shared-memory stages (full/empty mbarriers) and two TMEM
 // accumulators (tmem_full/tmem_empty) so the epilogue of tile i overlaps the
 // main loop of tile i+1.
@@ -42,8 +42,8 @@ namespace {
 constexpr int BM = 128;   // tile rows (MMA M, TMEM lanes)
 constexpr int BK = 64;    // K per stage: one 128-byte swizzle row of bf16
 constexpr int UK = 16;    // K of one tcgen05.mma kind::f16
-constexpr int NUM_THREADS = 320;
-constexpr int EPI_WARPS = 8;
+constexpr int EPI_WARPS = 16;                    // four per TMEM lane quadrant
+constexpr int NUM_THREADS = 64 + 32 * EPI_WARPS;  // producer + MMA warps + epilogue
 constexpr int MAX_GROUPS = 136;
 
 struct Params {
@@ -243,16 +243,20 @@ struct Cfg {
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int BN_OUT = (EPI == EPI_SWIGLU) ? BN / 2 : BN;
-  static constexpr int HALF = BN_OUT / 2;               // columns per epilogue warp
-  static constexpr int CW = (HALF % 32 == 0) ? 32 : 16;  // columns per TMEM load (divides HALF)
-  static_assert(HALF % CW == 0 && CW % 16 == 0, "epilogue chunks must tile each half exactly");
+  // columns of a tile split among the warps of a lane quadrant: PARTS parts
+  // of PART columns (a multiple of the 16-column TMEM load)
+  static constexpr int PARTS = (BN_OUT % 64 == 0) ? 4 : ((BN_OUT % 48 == 0) ? 3 : ((BN_OUT % 32 == 0) ? 2 : 1));
+  static constexpr int PART = BN_OUT / PARTS;
+  static constexpr int CW = 16;  // columns per TMEM load
+  static_assert(PART % CW == 0, "epilogue chunks must tile each part exactly");
   static constexpr int TMEM_COLS = pow2_at_least(2 * BN);  // two accumulators
   static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8;
-  static constexpr int STG_PITCH = CW * 2 + 16;          // bytes per staged row (padded: conflict-free)
+  static constexpr int STG_PITCH = CW * 2 + 16;          // bytes per staged row (padded)
   static constexpr int STG_BYTES = EPI_WARPS * 32 * STG_PITCH;
   static constexpr int OFF_INTS = 132;  // expert offsets of EPI_REPLICATE's relative mode (<= 128 + 1, padded)
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES + 16 + 2 * (MAX_GROUPS + 1) * 4 + OFF_INTS * 4 +
                               STG_BYTES;
+  static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
 template <int BN, int EPI, int STAGES>
@@ -436,8 +440,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // ---------------------------------------------------------------- epilogue
-    const int q = warp & 3;          // TMEM lane quadrant this warp may access
-    const int half = (warp - 2) >> 2;  // which half of the tile's columns
+    const int q = warp & 3;              // TMEM lane quadrant this warp may access
+    const int part = (warp - 2) >> 2;    // which part of the tile's columns
     const int row_in_tile = q * 32 + lane;
     int it = 0;
     int cursor = 0;
@@ -445,8 +449,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const TileCoord tc = decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
-      if (!mbar_wait(smem_u32(&tfull[acc]), acc_phase, budget, abort_flag)) break;
-      tc_fence_after();
+      // Row metadata first: its global loads overlap the tile's main loop.
       const int mg = p.offsets ? (p.offsets[tc.g + 1] - p.offsets[tc.g]) : p.M;
       const int local = tc.m_blk * BM + row_in_tile;
       const bool valid = local < mg;
@@ -474,25 +477,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
+      if (!mbar_wait(smem_u32(&tfull[acc]), acc_phase, budget, abort_flag)) break;
+      tc_fence_after();
       const uint32_t t_row = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
       // Each chunk of 32 rows x CW columns is staged in shared memory (thread =
-      // row) and written back with 4 lanes per row segment, so a warp store
-      // covers CW*2/16 ... contiguous 16-byte pieces of 32/(CW/8) rows.
+      // row) and written back with CW/8 lanes per row, so a warp store writes
+      // whole 32-byte sectors of 16 rows instead of 16-byte pieces of 32 rows.
       uint8_t* stg = stg_all + (warp - 2) * 32 * C::STG_PITCH;
       constexpr int SEGS = C::CW / 8;           // 16-byte segments per row
       constexpr int ROWS_PER_PASS = 32 / SEGS;  // rows a warp store covers
       // Two chunks' TMEM loads are issued before one wait (half as many waits);
-      // a half with an odd number of chunks ends on a single chunk.
-      constexpr int NCH = C::HALF / C::CW;
+      // a part with an odd number of chunks ends on a single chunk.  Warps
+      // beyond PARTS (narrow tiles) have no columns.
+      constexpr int NCH = C::PART / C::CW;
+      const int nch_mine = part < C::PARTS ? NCH : 0;
       uint32_t rv[2][C::CW], ru[2][C::CW];
 #pragma unroll 1
-      for (int ci = 0; ci < NCH; ++ci) {
-        const int c0 = half * C::HALF + ci * C::CW;
+      for (int ci = 0; ci < nch_mine; ++ci) {
+        const int c0 = part * C::PART + ci * C::CW;
         const int slot = ci & 1;
         if (slot == 0) {
           tmem_ld_nw<C::CW>(t_row + c0, rv[0]);
           if (EPI == EPI_SWIGLU) tmem_ld_nw<C::CW>(t_row + c0 + BN / 2, ru[0]);
-          if (ci + 1 < NCH) {
+          if (ci + 1 < nch_mine) {
             tmem_ld_nw<C::CW>(t_row + c0 + C::CW, rv[1]);
             if (EPI == EPI_SWIGLU) tmem_ld_nw<C::CW>(t_row + c0 + C::CW + BN / 2, ru[1]);
           }
