@@ -107,6 +107,8 @@ def kernel_work(cfg, name: str):
         return 2.0 * T * d * r, es * (T * d + r * d + T * r)
     if name == "lr_decode":
         return 2.0 * T * r * d, es * (T * r + d * r + T * d)
+    if name == "lr_codec":
+        return 4.0 * T * d * r, es * (T * d + 2 * r * d + T * r + n * d)
     if name == "gate_topk":
         return 2.0 * T * d * (E + K), es * T * d + 4 * (E + K) * d + 8 * n
     if name == "gather_rows":

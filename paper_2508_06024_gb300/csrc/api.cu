@@ -622,7 +622,28 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   // positions, and to the tail rows the shared experts read).
   const void* shared_a = xa;
   long long shared_a_rows = n + T, shared_a_base = n;
-  if (desc->r > 0) {
+  if (desc->r > 0 && routed && codec_fused_supported(desc->d, desc->r)) {
+    // encoder and decoder in one kernel; Z stays on chip between them
+    CodecArgs ca{};
+    ca.X = X;
+    ca.V_enc = w->V_enc;
+    ca.V_dec = w->V_dec;
+    ca.Z = zbuf;
+    ca.out = xa;
+    ca.T = desc->T;
+    ca.d = desc->d;
+    ca.r = desc->r;
+    ca.k = desc->k;
+    ca.E = desc->E;
+    ca.rel = inv_perm;
+    ca.counts = counts;
+    ca.topk_idx = topk_idx;
+    ca.perm_out = perm;
+    ca.offsets_out = offsets;
+    ca.self_row_base = desc->n_shared > 0 ? n : -1;
+    ca.timeout_cycles = default_timeout_cycles();
+    EC2MOE_CUDA(launch_codec_fused(ca, stream));
+  } else if (desc->r > 0) {
     EC2MOE_CUDA(run_codec(desc, true, X, w->V_enc, zbuf, stream));
     EC2MOE_CUDA(run_codec(desc, false, zbuf, w->V_dec, xa, stream, inv_perm, desc->n_shared > 0 ? n : -1, rel));
   } else {
@@ -654,9 +675,10 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
 
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream) {
   if (cudaStreamSynchronize(stream) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  unsigned int word = 0;
+  unsigned int word = 0, word2 = 0;
   if (read_tc_error(&word) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  return word ? EC2MOE_ERR_TIMEOUT : EC2MOE_OK;
+  if (read_codec_error(&word2) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  return (word | word2) ? EC2MOE_ERR_TIMEOUT : EC2MOE_OK;
 }
 
 int32_t ec2moe_last_launch_count(void) { return launch_count(); }

@@ -2,6 +2,7 @@
 // Nothing here is exported; the public ABI is include/ec2moe.h.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -141,6 +142,33 @@ struct GemmArgs {
 };
 cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s);    // bf16, tcgen05
 cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s);  // fp32, CUDA cores
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix: box 64 columns x
+// box_rows rows, 128-byte swizzle, zero fill out of bounds (cached).
+bool make_tensor_map_bf16(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows);
+
+// Fused low-rank codec of the layer path (bf16): Z = X V_enc^T (stored), then
+// X_hat = Z V_dec^T written straight into expert order with relative
+// placement (see EPI_REPLICATE's relative mode), plus the tail rows
+// [self_row_base + t] when self_row_base >= 0.  Needs r in {128, 256}.
+struct CodecArgs {
+  const void* X;
+  const void* V_enc;
+  const void* V_dec;
+  void* Z;        // [T, r] out
+  void* out;      // expert-ordered rows, pitch d
+  int T, d, r, k, E;
+  const int32_t* rel;      // [T*k] rows relative to each expert's first row
+  const int32_t* counts;   // [E]
+  const int32_t* topk_idx; // [T*k]
+  int32_t* perm_out;       // [T*k]
+  int32_t* offsets_out;    // [E+1]
+  long long self_row_base;
+  long long timeout_cycles;
+};
+bool codec_fused_supported(int d, int r);
+cudaError_t launch_codec_fused(const CodecArgs& a, cudaStream_t s);
+cudaError_t read_codec_error(unsigned int* word);
+
 // Reads and clears the tensor-core kernels' device error word (synchronous).
 cudaError_t read_tc_error(unsigned int* word);
 long long default_timeout_cycles();

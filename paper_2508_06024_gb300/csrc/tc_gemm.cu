@@ -32,12 +32,15 @@
 
 #include "common.cuh"
 #include "internal.h"
+#include "tc_ptx.cuh"
 
 namespace ec2moe {
 
 __device__ unsigned int g_tc_error;  // bit 0: a bounded wait timed out
 
 namespace {
+
+using namespace tc;
 
 constexpr int BM = 128;   // tile rows (MMA M, TMEM lanes)
 constexpr int BK = 64;    // K per stage: one 128-byte swizzle row of bf16
@@ -65,161 +68,6 @@ struct Params {
   long long timeout;
   int n_tiles_n;
 };
-
-// ------------------------------------------------------------------ PTX wrappers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}\n"
-      : "=r"(ok)
-      : "r"(bar), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Bounded wait.  Returns false when the budget ran out or another role of the
-// CTA already aborted (it then also raises the abort flag and the error word).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long long budget, volatile int* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
-  while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if (*abort_flag) return false;
-    if (clock64() - t0 > budget) {
-      *abort_flag = 1;
-      atomicOr(&g_tc_error, 1u);
-      return false;
-    }
-  }
-}
-// Wait used while draining after an abort: bounded, ignores the abort flag.
-__device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity, long long budget) {
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > budget) return;
-  }
-}
-
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* tm, int x, int y, uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
-      : "memory");
-}
-__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {
-  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// Shared-memory matrix descriptor (tcgen05 format) for a K-major operand tile
-// stored as rows of 128 bytes with the 128-byte swizzle, 8-row atoms 1024 bytes
-// apart.  Fields: start address >> 4 (bits 0-13), leading byte offset >> 4
-// (16-29, unused for swizzled K-major), stride byte offset >> 4 (32-45),
-// descriptor version 1 (46-47), base offset 0 (49-51), swizzle mode 2 =
-// 128-byte (61-63).
-__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
-  d |= static_cast<uint64_t>(1) << 16;
-  d |= static_cast<uint64_t>(1024 >> 4) << 32;
-  d |= static_cast<uint64_t>(1) << 46;
-  d |= static_cast<uint64_t>(2) << 61;
-  return d;
-}
-// Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator (bits 4-5
-// = 1), A and B bf16 (bits 7-9 and 10-12 = 1), both K-major (bits 15, 16 = 0),
-// N >> 3 in bits 17-22, M >> 4 in bits 24-28.
-__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n) {
-  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
-         (static_cast<uint32_t>(m >> 4) << 24);
-}
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t da, uint64_t db, uint32_t idesc, uint32_t accum) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
-      "l"(da), "l"(db), "r"(idesc), "r"(accum)
-      : "memory");
-}
-__device__ __forceinline__ void umma_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
-}
-// 32 lanes x 32 columns of 32-bit TMEM words: thread i of the warp receives
-// columns [col, col+32) of TMEM lane (quadrant base + i).
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
-  uint32_t r[16];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-template <int CW>
-__device__ __forceinline__ void tmem_ld(uint32_t taddr, float* v) {
-  if (CW == 32) tmem_ld32(taddr, v);
-  else tmem_ld16(taddr, v);
-}
-
-// Issue-only TMEM loads (the caller waits with tmem_wait once for several).
-__device__ __forceinline__ void tmem_ld32_nw(uint32_t taddr, uint32_t* r) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_ld16_nw(uint32_t taddr, uint32_t* r) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-      : "r"(taddr));
-}
-template <int CW>
-__device__ __forceinline__ void tmem_ld_nw(uint32_t taddr, uint32_t* r) {
-  if (CW == 32) tmem_ld32_nw(taddr, r);
-  else tmem_ld16_nw(taddr, r);
-}
-__device__ __forceinline__ void tmem_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
 // ------------------------------------------------------------------ tile schedule
 struct TileCoord {
@@ -363,7 +211,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                           tc.m_blk * BM;
         const int b_row = tc.g * p.b_group_rows + tc.n_blk * C::BN_OUT;
         for (int kb = 0; kb < num_kb; ++kb) {
-          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1u, budget, abort_flag)) {
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1u, budget, abort_flag, &g_tc_error)) {
             ok = false;
             break;
           }
@@ -394,6 +242,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
       constexpr uint32_t IDESC = idesc_bf16(BM, BN);
+      constexpr uint64_t DA_STAGE = C::A_BYTES >> 4;
+      constexpr uint64_t DB_STAGE = C::B_BYTES >> 4;
+      const uint64_t da0 = sdesc_sw128(smem_u32(sA));
+      const uint64_t db0 = sdesc_sw128(smem_u32(sB));
+      const uint32_t full0 = smem_u32(&full[0]);
+      const uint32_t empty0 = smem_u32(&empty[0]);
       int stage = 0;
       uint32_t phase = 0;
       int it = 0;
@@ -403,27 +257,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         (void)decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
-        if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, budget, abort_flag)) {
+        if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, budget, abort_flag, &g_tc_error)) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
         for (int kb = 0; kb < num_kb; ++kb) {
-          if (!mbar_wait(smem_u32(&full[stage]), phase, budget, abort_flag)) {
+          if (!mbar_wait(full0 + 8u * stage, phase, budget, abort_flag, &g_tc_error)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(sA + stage * C::A_BYTES);
-          const uint32_t b0 = smem_u32(sB + stage * C::B_BYTES);
+          // Descriptors of this stage: the stage-0 descriptors plus the stage
+          // offset; each K = 16 step adds 32 bytes (2 in the address field).
+          // The address field (bits 0-13) cannot carry: shared addresses are
+          // below 256 KB.
+          const uint64_t da = da0 + static_cast<uint64_t>(stage) * DA_STAGE;
+          const uint64_t db = db0 + static_cast<uint64_t>(stage) * DB_STAGE;
+          umma_bf16(d_tmem, da, db, IDESC, kb != 0 ? 1u : 0u);
 #pragma unroll
-          for (int kk = 0; kk < BK / UK; ++kk) {
-            umma_bf16(d_tmem, sdesc_sw128(a0 + kk * UK * 2), sdesc_sw128(b0 + kk * UK * 2), IDESC,
-                      (kb | kk) != 0 ? 1u : 0u);
-          }
+          for (int kk = 1; kk < BK / UK; ++kk) umma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, IDESC, 1u);
           any = true;
-          umma_commit(smem_u32(&empty[stage]));
+          umma_commit(empty0 + 8u * stage);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
@@ -477,7 +333,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
-      if (!mbar_wait(smem_u32(&tfull[acc]), acc_phase, budget, abort_flag)) break;
+      if (!mbar_wait(smem_u32(&tfull[acc]), acc_phase, budget, abort_flag, &g_tc_error)) break;
       tc_fence_after();
       const uint32_t t_row = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
       // Each chunk of 32 rows x CW columns is staged in shared memory (thread =
@@ -745,6 +601,10 @@ int choose_bn(const GemmArgs& a, int epi) {
 }
 
 }  // namespace
+
+bool make_tensor_map_bf16(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+  return make_map(m, ptr, rows, cols, box_rows);
+}
 
 cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
   if (a.G < 1 || a.G > MAX_GROUPS || a.N % 32 != 0 || a.K % 8 != 0) return cudaErrorInvalidValue;
