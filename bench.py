@@ -210,6 +210,26 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+# ------------------------------------------------------------------ multi-rank helpers
+def reduce_max(values, device=None):
+    """Element-wise max of a list of floats over all ranks (identity when not distributed).
+
+    Tokens are independent, so ranks share no data; this reduction of the
+    timings is the only collective the benchmark uses."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return list(values)
+    t = torch.tensor(list(values), dtype=torch.float64, device=device or "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return t.tolist()
+
+
+def whole_job_tokens_per_s(world: int, tokens_per_rank: int, max_ms_per_step: float) -> float:
+    """Weak scaling: every rank processes its own batch; the slowest rank sets the step time."""
+    return world * tokens_per_rank / (max_ms_per_step * 1e-3)
+
+
 # ------------------------------------------------------------------ reference arm (fp64 oracle on CPU)
 def oracle_sample_step(cfg, o, rows):
     from oracle import ec2moe_oracle as orc
@@ -401,11 +421,9 @@ def run_ours(args):
             per_kernel.setdefault(name, []).append(ms)
     C.ec2moe_profile_reset()
 
-    total_ms = torch.tensor([sum(step_ms), sum(e2e_ms)], dtype=torch.float64, device=dev)
-    if world > 1:
-        dist.all_reduce(total_ms, op=dist.ReduceOp.MAX)
-    t_step = total_ms[0].item() / args.steps
-    t_e2e = total_ms[1].item() / args.steps
+    tot_step, tot_e2e = reduce_max([sum(step_ms), sum(e2e_ms)], device=dev)
+    t_step = tot_step / args.steps
+    t_e2e = tot_e2e / args.steps
     if rank != 0:
         if world > 1:
             dist.destroy_process_group()
@@ -431,7 +449,7 @@ def run_ours(args):
         cpu = {"value": round(tps, 2), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
                "sample": desc}
 
-    value = world * cfg.T / (t_step * 1e-3)
+    value = whole_job_tokens_per_s(world, cfg.T, t_step)
     es = 2 if cfg.dtype == 1 else 4
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
@@ -446,7 +464,7 @@ def run_ours(args):
         "kernels": {n: dict(kern[n], bound=others[n]["bound"], achieved=others[n]["achieved"],
                             unit=others[n]["unit"], frac=others[n]["frac"]) for n in sorted(kern)},
         "cpu_baseline": cpu,
-        "e2e": {"value": round(world * cfg.T / (t_e2e * 1e-3), 1), "unit": "tokens/s",
+        "e2e": {"value": round(whole_job_tokens_per_s(world, cfg.T, t_e2e), 1), "unit": "tokens/s",
                 "h2d_bytes_per_step": cfg.T * cfg.d * es, "d2h_bytes_per_step": cfg.T * cfg.d * es,
                 "ms_per_step": round(t_e2e, 5)},
         "gpu_launches": launches_per_step * args.steps,

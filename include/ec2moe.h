@@ -235,6 +235,17 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
  * error. */
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream);
 
+/* Budget, in SM clock cycles, of every bounded wait inside the tensor-core
+ * kernels of later calls (process-wide; default 4e9, about two seconds).  A
+ * wait that runs out makes its CTA stop, wait (with a fixed one-second
+ * budget) for the copies and MMAs it started, free its tensor memory and
+ * return; ec2moe_last_device_error then reports EC2MOE_ERR_TIMEOUT and the
+ * context stays usable.  A budget of 0 makes every wait that is not already
+ * satisfied give up at once, which is how failure handling is exercised
+ * without a real fault.  Negative values return EC2MOE_ERR_INVALID_ARG. */
+ec2moe_status ec2moe_set_wait_budget(int64_t cycles);
+int64_t ec2moe_get_wait_budget(void);
+
 /* Number of kernels the last successful call on this host thread enqueued. */
 int32_t ec2moe_last_launch_count(void);
 

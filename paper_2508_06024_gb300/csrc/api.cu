@@ -683,6 +683,14 @@ ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream) {
 
 int32_t ec2moe_last_launch_count(void) { return launch_count(); }
 
+ec2moe_status ec2moe_set_wait_budget(int64_t cycles) {
+  if (cycles < 0) return EC2MOE_ERR_INVALID_ARG;
+  set_timeout_cycles(cycles == 0 ? 0 : cycles);
+  return EC2MOE_OK;
+}
+
+int64_t ec2moe_get_wait_budget(void) { return default_timeout_cycles(); }
+
 ec2moe_status ec2moe_profile_enable(int32_t enable) {
   std::lock_guard<std::mutex> lock(g_prof_mu);
   g_prof_on = enable != 0;

@@ -174,7 +174,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       if (!ok || *abort_flag) {
         for (int s = 0; s < C::STAGES; ++s)
-          if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, budget);
+          if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, DRAIN_CYCLES);
       }
     }
   } else if (warp == 1) {
@@ -232,7 +232,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (ok) umma_commit(smem_u32(xfull));
       if ((!ok || *abort_flag) && any) {
         umma_commit(smem_u32(drain));
-        mbar_drain(smem_u32(drain), 0, budget);
+        mbar_drain(smem_u32(drain), 0, DRAIN_CYCLES);
       }
     }
   } else {

@@ -172,5 +172,6 @@ cudaError_t read_codec_error(unsigned int* word);
 // Reads and clears the tensor-core kernels' device error word (synchronous).
 cudaError_t read_tc_error(unsigned int* word);
 long long default_timeout_cycles();
+void set_timeout_cycles(long long cycles);
 
 }  // namespace ec2moe

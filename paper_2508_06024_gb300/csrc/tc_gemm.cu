@@ -28,6 +28,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <mutex>
 
 #include "common.cuh"
@@ -235,7 +236,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if (!ok || *abort_flag) {
         // Let every copy this CTA started land before shared memory is released.
         for (int s = 0; s < STAGES; ++s)
-          if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, budget);
+          if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, DRAIN_CYCLES);
       }
     }
   } else if (warp == 1) {
@@ -291,7 +292,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       if ((!ok || *abort_flag) && any) {
         // All MMAs issued so far must finish before TMEM is freed.
         umma_commit(smem_u32(drain));
-        mbar_drain(smem_u32(drain), 0, budget);
+        mbar_drain(smem_u32(drain), 0, DRAIN_CYCLES);
       }
     }
   } else {
@@ -626,7 +627,12 @@ cudaError_t read_tc_error(unsigned int* word) {
   return cudaMemcpyToSymbol(g_tc_error, &zero, sizeof(unsigned int));
 }
 
-// About two seconds at the GB300's maximum SM clock.
-long long default_timeout_cycles() { return 4000000000LL; }
+// About two seconds at the GB300's maximum SM clock unless changed with
+// ec2moe_set_wait_budget.
+namespace {
+std::atomic<long long> g_wait_budget{4000000000LL};
+}
+long long default_timeout_cycles() { return g_wait_budget.load(); }
+void set_timeout_cycles(long long cycles) { g_wait_budget.store(cycles); }
 
 }  // namespace ec2moe

@@ -50,6 +50,12 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, long lo
     }
   }
 }
+// Budget of the drain waits after an abort (about one second at the maximum
+// SM clock), independent of the caller-set wait budget: copies and MMAs a
+// CTA started must land before its shared memory and TMEM are released,
+// however short the budget that triggered the abort was.
+constexpr long long DRAIN_CYCLES = 2000000000LL;
+
 // Wait used while draining after an abort: bounded, ignores the abort flag.
 __device__ __forceinline__ void mbar_drain(uint32_t bar, uint32_t parity, long long budget) {
   const long long t0 = clock64();

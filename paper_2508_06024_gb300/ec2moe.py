@@ -39,7 +39,8 @@ EXPORTED = [
     "ec2moe_gate", "ec2moe_route", "ec2moe_experts", "ec2moe_shared_experts", "ec2moe_combine",
     "ec2moe_lr_encode", "ec2moe_lr_decode", "ec2moe_layer_forward", "ec2moe_last_device_error",
     "ec2moe_last_launch_count", "ec2moe_status_string", "ec2moe_profile_enable", "ec2moe_profile_count",
-    "ec2moe_profile_read", "ec2moe_profile_reset", "ec2moe_route_noalloc",
+    "ec2moe_profile_read", "ec2moe_profile_reset", "ec2moe_route_noalloc", "ec2moe_set_wait_budget",
+    "ec2moe_get_wait_budget",
 ]
 
 
@@ -87,6 +88,8 @@ _SIGS = {
     "ec2moe_profile_read": (ctypes.c_int, [ctypes.c_int32, ctypes.POINTER(ctypes.c_char_p),
                                            ctypes.POINTER(ctypes.c_float)]),
     "ec2moe_profile_reset": (None, []),
+    "ec2moe_set_wait_budget": (ctypes.c_int, [ctypes.c_int64]),
+    "ec2moe_get_wait_budget": (ctypes.c_int64, []),
 }
 
 
@@ -252,3 +255,11 @@ def ec2moe_profile_read(i: int):
 
 def ec2moe_profile_reset() -> None:
     load().ec2moe_profile_reset()
+
+
+def ec2moe_set_wait_budget(cycles: int) -> None:
+    _check(load().ec2moe_set_wait_budget(int(cycles)), "ec2moe_set_wait_budget")
+
+
+def ec2moe_get_wait_budget() -> int:
+    return int(load().ec2moe_get_wait_budget())
