@@ -522,6 +522,126 @@ __global__ void __launch_bounds__(SL_THREADS) gate_slices_kernel(const KParams p
   }
 }
 
+// Gate for gate matrices that do not fit in shared memory (many experts and a
+// wide d_model): a register-tiled fp32 product of a 64-token tile with all
+// O = E + K gate rows, d_model streamed through shared memory 32 columns at a
+// time (the next chunk is loaded into registers while the current one is
+// used).  Thread (q, g) owns tokens 4q .. 4q+3 and gate rows OPT*g .. +OPT-1.
+// Each dot product is summed in 256-column partials that are then added,
+// keeping the fp32 rounding close to that of a short sum.  One warp per token
+// then takes the softmax / Top-k decision; the layer path also reserves the
+// tile's rows per expert.
+constexpr int GT_BM = 64;
+constexpr int GT_KC = 32;
+constexpr int GT_PARTIAL = 256;
+
+template <typename TX, int OPT>
+__global__ void __launch_bounds__(SL_THREADS) gate_tiled_kernel(const KParams p) {
+  constexpr int OP = 16 * OPT;
+  __shared__ __align__(16) float sX[GT_KC][GT_BM + 4];  // k-major activations
+  __shared__ __align__(16) float sW[GT_KC][OP + 4];     // k-major gate rows
+  __shared__ int s_base[128];
+  extern __shared__ float smem_f[];
+  const int nglob = (p.K == 1) ? 0 : p.K;
+  const int O = p.E + nglob;
+  float* sLog = smem_f;                                  // [GT_BM][O]
+  int* sIdx = reinterpret_cast<int*>(sLog + GT_BM * O);  // [GT_BM * k]
+  const int tq = threadIdx.x >> 4;  // token quad
+  const int og = threadIdx.x & 15;  // gate-row group
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_trigger();
+  pdl_wait();
+  const TX* X = reinterpret_cast<const TX*>(p.X);
+  const int n_tiles = (p.T + GT_BM - 1) / GT_BM;
+  const int nk = p.d / GT_KC;
+  // staging assignment: X chunk = 64 tokens x 32 columns (8 per thread);
+  // W chunk = OP rows x 32 columns (OP * 8 float4, up to 3 per thread)
+  const int xr = threadIdx.x >> 2, xc = (threadIdx.x & 3) * 8;
+  for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    const int t0 = tile * GT_BM;
+    float acc[4][OPT], part[4][OPT];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < OPT; ++j) acc[i][j] = part[i][j] = 0.0f;
+    float xv[8];
+    float4 wv[3];
+    auto load_chunk = [&](int kc) {
+      const int tok = t0 + xr;
+      if (tok < p.T) load8(X + (size_t)tok * p.d + kc * GT_KC + xc, xv);
+      else
+#pragma unroll
+        for (int q = 0; q < 8; ++q) xv[q] = 0.0f;
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        const int i = threadIdx.x + u * SL_THREADS;  // float4 index in the [OP][8] chunk
+        const int o = i >> 3, c = (i & 7) * 4;
+        wv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (i < OP * 8 && o < O) {
+          const float* src = o < p.E ? p.W_local + (size_t)o * p.d : p.W_global + (size_t)(o - p.E) * p.d;
+          wv[u] = *reinterpret_cast<const float4*>(src + kc * GT_KC + c);
+        }
+      }
+    };
+    load_chunk(0);
+    for (int kc = 0; kc < nk; ++kc) {
+      __syncthreads();
+#pragma unroll
+      for (int q = 0; q < 8; ++q) sX[xc + q][xr] = xv[q];
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        const int i = threadIdx.x + u * SL_THREADS;
+        if (i < OP * 8) {
+          const int o = i >> 3, c = (i & 7) * 4;
+          sW[c + 0][o] = wv[u].x;
+          sW[c + 1][o] = wv[u].y;
+          sW[c + 2][o] = wv[u].z;
+          sW[c + 3][o] = wv[u].w;
+        }
+      }
+      __syncthreads();
+      if (kc + 1 < nk) load_chunk(kc + 1);  // in flight during this chunk's FMAs
+#pragma unroll 8
+      for (int k = 0; k < GT_KC; ++k) {
+        const float4 x4 = *reinterpret_cast<const float4*>(&sX[k][tq * 4]);
+        float w[OPT];
+#pragma unroll
+        for (int j = 0; j < OPT; ++j) w[j] = sW[k][og * OPT + j];
+#pragma unroll
+        for (int j = 0; j < OPT; ++j) {
+          part[0][j] = fmaf(x4.x, w[j], part[0][j]);
+          part[1][j] = fmaf(x4.y, w[j], part[1][j]);
+          part[2][j] = fmaf(x4.z, w[j], part[2][j]);
+          part[3][j] = fmaf(x4.w, w[j], part[3][j]);
+        }
+      }
+      if (((kc + 1) * GT_KC) % GT_PARTIAL == 0 || kc + 1 == nk) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int j = 0; j < OPT; ++j) {
+            acc[i][j] += part[i][j];
+            part[i][j] = 0.0f;
+          }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < OPT; ++j) {
+        const int o = og * OPT + j;
+        if (o < O) sLog[(tq * 4 + i) * O + o] = acc[i][j] + (o < p.E ? p.b_local[o] : p.b_global[o - p.E]);
+      }
+    __syncthreads();
+    for (int jj = warp; jj < GT_BM; jj += SL_THREADS / 32) {
+      const int tok = t0 + jj;
+      if (tok < p.T) decide_token_warp(p, sLog + jj * O, tok, lane, p.route_counts ? sIdx + jj * p.k : nullptr);
+    }
+    __syncthreads();
+    if (p.route_counts) route_tile(p, tile, GT_BM, sIdx, s_base);
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed) {
@@ -600,6 +720,36 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* rout
 #undef EC2MOE_SLICES
       return cudaGetLastError();
     }
+  }
+  // Register-tiled kernel when the gate rows do not fit in shared memory.
+  if (a.d % GT_KC == 0 && O <= 144) {
+    const int opt = O <= 80 ? 5 : 9;
+    const size_t smem = (size_t)GT_BM * O * 4 + (size_t)GT_BM * a.k * 4;
+    const long long tiles = (a.T + GT_BM - 1) / GT_BM;
+    long long blocks = tiles < (long long)sm_count() * 2 ? tiles : (long long)sm_count() * 2;
+    if (blocks < 1) blocks = 1;
+    if (a.route_counts && a.route_rel) {
+      p.route_counts = a.route_counts;
+      p.route_rel = a.route_rel;
+      e = cudaMemsetAsync(a.route_counts, 0, sizeof(int32_t) * a.E, s);
+      if (e != cudaSuccess) return e;
+      if (routed) *routed = true;
+    }
+    KernelScope ks("gate_topk", s);
+#define EC2MOE_TILED(TX, OPTV)                                                                               \
+  do {                                                                                                      \
+    e = ensure_smem_attr(reinterpret_cast<const void*>(gate_tiled_kernel<TX, OPTV>), (int)smem);            \
+    if (e != cudaSuccess) return e;                                                                         \
+    e = launch_kernel(gate_tiled_kernel<TX, OPTV>, dim3((int)blocks), dim3(SL_THREADS), smem, s, p);        \
+    if (e != cudaSuccess) return e;                                                                         \
+  } while (0)
+    if (bf16) {
+      if (opt == 5) EC2MOE_TILED(__nv_bfloat16, 5); else EC2MOE_TILED(__nv_bfloat16, 9);
+    } else {
+      if (opt == 5) EC2MOE_TILED(float, 5); else EC2MOE_TILED(float, 9);
+    }
+#undef EC2MOE_TILED
+    return cudaGetLastError();
   }
   const size_t base = (size_t)(WARPS * TPW * MAXO + WARPS * TPW * 32) * sizeof(float);
   const size_t wbytes = (size_t)O * a.d * sizeof(float);
