@@ -111,6 +111,9 @@ def kernel_work(cfg, name: str):
         return 4.0 * T * d * r, es * (T * d + 2 * r * d + T * r + n * d)
     if name == "gate_topk":
         return 2.0 * T * d * (E + K), es * T * d + 4 * (E + K) * d + 8 * n
+    if name == "gate_prep":
+        n_pad = -(-(E + K) // 16) * 16
+        return 0.0, 4 * (E + K) * d + 2 * 3 * n_pad * d + 4 * E
     if name == "gather_rows":
         return 0.0, 2 * es * n * d + 4 * n
     if name == "combine":

@@ -193,7 +193,7 @@ ec2moe_status check_mask(const ec2moe_layer_desc* d, const uint8_t* mask, uint32
 
 // Workspace of ec2moe_layer_forward, each region 256-byte aligned.
 struct LayerWs {
-  size_t z, xa, h, slot, shared, perm, inv_perm, offsets, blk, total;
+  size_t z, xa, h, slot, shared, perm, inv_perm, offsets, blk, wsplit, total;
 };
 LayerWs layer_ws(const ec2moe_layer_desc* d) {
   LayerWs w{};
@@ -216,6 +216,7 @@ LayerWs layer_ws(const ec2moe_layer_desc* d) {
   w.inv_perm = take(T * k * 4);
   w.offsets = take((d->E + 1) * 4);
   w.blk = take((size_t)route_blocks((long long)T * k) * d->E * 4);
+  w.wsplit = take(gate_split_bytes(d->E, d->n_groups, d->d, is_bf16(d)));
   w.total = off;
   return w;
 }
@@ -605,6 +606,7 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   if (bf) {
     ga.route_counts = counts;
     ga.route_rel = inv_perm;
+    if (gate_split_bytes(desc->E, desc->n_groups, desc->d, bf)) ga.w_split = ws + L.wsplit;
   }
   bool routed = false;
   EC2MOE_CUDA(launch_gate(ga, bf, stream, &routed));
@@ -675,10 +677,11 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
 
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream) {
   if (cudaStreamSynchronize(stream) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  unsigned int word = 0, word2 = 0;
+  unsigned int word = 0, word2 = 0, word3 = 0;
   if (read_tc_error(&word) != cudaSuccess) return EC2MOE_ERR_CUDA;
   if (read_codec_error(&word2) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  return (word | word2) ? EC2MOE_ERR_TIMEOUT : EC2MOE_OK;
+  if (read_gate_error(&word3) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  return (word | word2 | word3) ? EC2MOE_ERR_TIMEOUT : EC2MOE_OK;
 }
 
 int32_t ec2moe_last_launch_count(void) { return launch_count(); }

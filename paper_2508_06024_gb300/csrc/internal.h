@@ -75,7 +75,14 @@ struct GateArgs {
   // first row).  Consumers place rows at offsets[e] + route_rel[i].
   int32_t* route_counts;
   int32_t* route_rel;
+  // Optional workspace of gate_split_bytes() bytes (256-byte aligned): with
+  // it the tensor-core gate reads the gate rows pre-split into three bf16
+  // terms by a small kernel launched first; nullptr: the gate kernel splits
+  // them itself.
+  void* w_split;
 };
+// Bytes of the prepared split gate rows (0 when the tensor-core gate does not apply).
+size_t gate_split_bytes(int E, int K, int d, bool bf16);
 // Launches the gate; with the routing fields set, also fills them when the
 // fused path applies (*routed = true), else gate only.
 cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed = nullptr);
@@ -145,6 +152,8 @@ cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s);  // fp
 // 2-D bf16 tensor map over a row-major [rows, cols] matrix: box 64 columns x
 // box_rows rows, 128-byte swizzle, zero fill out of bounds (cached).
 bool make_tensor_map_bf16(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows);
+// 2-D fp32 tensor map, box 64 columns x box_rows rows, no swizzle (cached).
+bool make_tensor_map_f32(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows);
 
 // Fused low-rank codec of the layer path (bf16): Z = X V_enc^T (stored), then
 // X_hat = Z V_dec^T written straight into expert order with relative
@@ -168,6 +177,8 @@ struct CodecArgs {
 bool codec_fused_supported(int d, int r);
 cudaError_t launch_codec_fused(const CodecArgs& a, cudaStream_t s);
 cudaError_t read_codec_error(unsigned int* word);
+// Reads and clears the tensor-core gate's device error word (synchronous).
+cudaError_t read_gate_error(unsigned int* word);
 
 // Reads and clears the tensor-core kernels' device error word (synchronous).
 cudaError_t read_tc_error(unsigned int* word);

@@ -438,24 +438,32 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-bool encode_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows);
+// Map kinds: bf16 with the 128-byte swizzle, or fp32 unswizzled (rows of
+// 64 x 4 = 256 bytes in shared memory).
+enum MapKind { MAP_BF16_SW128 = 0, MAP_F32_PLAIN = 1 };
 
-// Encoded tensor maps are cached by (device, address, shape, box): encoding
-// costs host time on every launch otherwise.  A map only describes an address
-// and a layout, so a hit stays valid even if the memory was reallocated.
+bool encode_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows, int kind);
+
+// Encoded tensor maps are cached by (device, address, shape, box, kind):
+// encoding costs host time on every launch otherwise.  A map only describes
+// an address and a layout, so a hit stays valid even if the memory was
+// reallocated.
 struct MapKey {
   int dev;
   const void* ptr;
   long long rows, cols;
   int box_rows;
+  int kind;
   bool operator==(const MapKey& o) const {
-    return dev == o.dev && ptr == o.ptr && rows == o.rows && cols == o.cols && box_rows == o.box_rows;
+    return dev == o.dev && ptr == o.ptr && rows == o.rows && cols == o.cols && box_rows == o.box_rows &&
+           kind == o.kind;
   }
 };
 
-// 2-D bf16 tensor map over a row-major [rows, cols] matrix, box = 64 columns x box_rows
-// rows, 128-byte swizzle, zero fill out of bounds.
-bool make_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+// 2-D tensor map over a row-major [rows, cols] matrix, box = 64 columns x
+// box_rows rows, zero fill out of bounds.
+bool make_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows,
+              int kind = MAP_BF16_SW128) {
   constexpr int SLOTS = 64;
   static std::mutex mu;
   static MapKey keys[SLOTS];
@@ -464,7 +472,7 @@ bool make_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, i
   static int next = 0;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;
-  const MapKey key{dev, ptr, rows, cols, box_rows};
+  const MapKey key{dev, ptr, rows, cols, box_rows, kind};
   {
     std::lock_guard<std::mutex> lock(mu);
     for (int i = 0; i < SLOTS; ++i)
@@ -473,7 +481,7 @@ bool make_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, i
         return true;
       }
   }
-  if (!encode_map(m, ptr, rows, cols, box_rows)) return false;
+  if (!encode_map(m, ptr, rows, cols, box_rows, kind)) return false;
   std::lock_guard<std::mutex> lock(mu);
   keys[next] = key;
   maps[next] = *m;
@@ -482,15 +490,17 @@ bool make_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, i
   return true;
 }
 
-bool encode_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+bool encode_map(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows, int kind) {
   auto fn = encode_fn();
   if (!fn) return false;
+  const bool f32 = kind == MAP_F32_PLAIN;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * 2};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(cols) * (f32 ? 4 : 2)};
   cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
-  CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+  CUresult r = fn(m, f32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                  const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  f32 ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
 }
@@ -604,7 +614,11 @@ int choose_bn(const GemmArgs& a, int epi) {
 }  // namespace
 
 bool make_tensor_map_bf16(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
-  return make_map(m, ptr, rows, cols, box_rows);
+  return make_map(m, ptr, rows, cols, box_rows, MAP_BF16_SW128);
+}
+
+bool make_tensor_map_f32(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows) {
+  return make_map(m, ptr, rows, cols, box_rows, MAP_F32_PLAIN);
 }
 
 cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {

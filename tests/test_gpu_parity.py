@@ -54,6 +54,12 @@ GATE_CASES = [
     # every allowed expert selected (k = |E_local|); a whole group masked out
     S.preset("tiny_fp32", n_allowed=2, k=2, seed=5),
     S.preset("switch_bf16", T=513, E=16, n_groups=4, k=3, n_allowed=5, seed=6),
+    # more token tiles than SMs (each CTA runs several tiles); d_model not a
+    # multiple of the 64-column stage; exactly 80 gate rows; 136 gate rows
+    S.preset("switch_bf16", T=20000, seed=17),
+    S.preset("switch_bf16", T=300, d=200, seed=16),
+    S.preset("finegrained_bf16", T=900, n_groups=16, k=4, seed=19),
+    S.preset("finegrained_bf16", T=700, E=128, n_groups=8, n_allowed=64, k=4, seed=15),
 ]
 
 
@@ -77,6 +83,37 @@ def test_gate_topk(cfg):
     keep = ref["gap_boundary"] >= TIE_GAP
     assert np.array_equal(np.bincount(gi[keep].ravel(), minlength=cfg.E),
                           np.bincount(ref["idx"][keep].ravel(), minlength=cfg.E))
+
+
+NONFINITE_CASES = [S.preset("tiny_fp32", seed=21), S.preset("switch_bf16", T=300, seed=22),
+                   S.preset("finegrained_bf16", T=300, seed=23),
+                   S.preset("finegrained_bf16", T=300, E=128, n_groups=8, n_allowed=64, k=4, seed=24)]
+
+
+@pytest.mark.parametrize("cfg", NONFINITE_CASES, ids=lambda c: f"{c.name}-E{c.E}")
+def test_gate_nonfinite_token_names_valid_experts(cfg):
+    """A token with NaN activations still gets k distinct allowed experts (the
+    lowest allowed ones, with NaN weights); the other tokens are unaffected."""
+    inp = S.make_inputs(cfg, device="cuda", with_experts=False)
+    bad = [0, cfg.T // 2, cfg.T - 1]
+    inp["X"][bad] = float("nan")
+    desc = desc_for(cfg)
+    idx = torch.full((cfg.T, cfg.k), -1, dtype=torch.int32, device="cuda")
+    w = torch.zeros((cfg.T, cfg.k), dtype=torch.float32, device="cuda")
+    C.ec2moe_gate(desc, inp["X"], inp["W_local"], inp["b_local"], inp["W_global"], inp["b_global"],
+                  inp["mask"].cpu(), idx, w)
+    torch.cuda.synchronize()
+    gi, gw = idx.cpu().numpy(), w.cpu().numpy()
+    allowed = np.flatnonzero(inp["mask"].cpu().numpy())
+    for t in bad:
+        assert sorted(gi[t].tolist()) == allowed[: cfg.k].tolist()
+        assert np.isnan(gw[t]).all()
+    good = np.setdiff1d(np.arange(cfg.T), bad)
+    inp["X"][bad] = 0.0
+    ref = _gate_ref(cfg, inp)
+    sub = {key: (v[good] if isinstance(v, np.ndarray) and v.shape[:1] == (cfg.T,) else v) for key, v in ref.items()}
+    n_cmp, n_excl = routing_check(gi[good], sub)
+    assert n_excl <= 2, n_excl
 
 
 ROUTE_CASES = [S.preset("tiny_fp32"), S.preset("switch_bf16"), S.preset("finegrained_bf16"),
@@ -146,6 +183,7 @@ LAYER_CASES = [
     (S.preset("switch_bf16", T=300, r=0, seed=9), None),
     (S.preset("switch_bf16", T=200, E=1, n_groups=1, n_allowed=1, k=1, seed=10), None),
     (S.preset("mixtral_bf16"), 256),
+    (S.preset("switch_bf16", T=20000, seed=18), 256),
     (S.preset("finegrained_bf16"), 256),
     (S.preset("finegrained_bf16", T=999, r=0, seed=11), None),
     (S.preset("decode_bf16", T=1, n_allowed=4, r=128, seed=1), None),
