@@ -253,7 +253,7 @@ int32_t ec2moe_last_launch_count(void);
  * bracketed by a pair of CUDA events recorded on its stream; records
  * accumulate until ec2moe_profile_reset.  Reading a record synchronises on its
  * stop event.  `name` receives a static string naming the launch
- * ("gate_topk", "route_count", "route_scatter", "gather_rows", "lr_encode",
+ * ("gate_prep", "gate_topk", "route_count", "route_scatter", "gather_rows", "lr_encode",
  * "lr_decode", "expert_up", "expert_down", "shared_up", "shared_down",
  * "combine"); `ms` its device duration.  Profiling is off by default and
  * costs nothing when off. */
@@ -261,6 +261,54 @@ ec2moe_status ec2moe_profile_enable(int32_t enable);
 int32_t ec2moe_profile_count(void);
 ec2moe_status ec2moe_profile_read(int32_t i, const char** name, float* ms);
 void ec2moe_profile_reset(void);
+
+/* ---------------------------------------------------------------------------
+ * Route-aware heuristic pipeline scheduler (Eq. 9-11 of the paper's pipeline
+ * optimisation).  Host code only: no device memory, no CUDA call, no stream.
+ * Every pointer below is a host pointer.
+ *
+ * ec2moe_schedule places n tasks, task i with computational complexity
+ * cost[i] = C(t_i) >= 0 and communication cost comm[i] = Comm(t_i) >= 0, on
+ * the End (location[i] = EC2MOE_END) or the Cloud (EC2MOE_CLOUD):
+ *   Eq. 10  P(t_i) = C(t_i) / (Comm(t_i) + eps)
+ *   Eq. 11  End if Load_end + C(t_i) <= T_end and P(t_i) >= beta, else Cloud,
+ * visiting the tasks in decreasing priority (ties to the lower index) and
+ * adding C(t_i) to Load_end (starting at load_end) for each End task and to
+ * Load_cloud (starting at load_cloud; reported only, Eq. 11 does not use it)
+ * for each Cloud task.  order[j] receives the j-th visited task (may be NULL);
+ * *load_end_out and *load_cloud_out the final loads (may be NULL).
+ * Errors: EC2MOE_ERR_INVALID_ARG for n < 0, NULL cost/comm/location when
+ * n > 0, a negative or NaN cost or comm, eps < 0 or NaN, or comm[i] + eps == 0
+ * for some i.  T_end and beta may be +/-infinity. */
+#define EC2MOE_END 0
+#define EC2MOE_CLOUD 1
+ec2moe_status ec2moe_schedule(int32_t n, const double* cost, const double* comm, double load_end,
+                              double load_cloud, double T_end, double beta, double eps, int32_t* location,
+                              int32_t* order, double* load_end_out, double* load_cloud_out);
+
+/* Eq. 9, the heuristic's objective for a placement:
+ *   sum_i alpha * ExecTime(t_i) + (1 - alpha) * Comm(t_i),
+ * with ExecTime(t_i) = cost[i] / rate_end on the End and cost[i] / rate_cloud
+ * on the Cloud, and Comm(t_i) paid by Cloud tasks only (a task run on the End
+ * transmits nothing).  Sums in task order.  Errors: EC2MOE_ERR_INVALID_ARG for
+ * n < 0, NULL arrays when n > 0, rates <= 0, a location other than
+ * EC2MOE_END / EC2MOE_CLOUD, or NULL `objective`. */
+ec2moe_status ec2moe_schedule_objective(int32_t n, const double* cost, const double* comm,
+                                        const int32_t* location, double rate_end, double rate_cloud,
+                                        double alpha, double* objective);
+
+/* Route-aware tasks from a layer's routing histogram (counts, host copy of
+ * the [E] output of ec2moe_route / ec2moe_layer_forward): one task per expert
+ * with rows, in expert order.  expert_of_task[j] is the expert of task j,
+ * cost[j] = 2 * rows * d * d_ff * (3 projections for SwiGLU, 2 for GELU) its
+ * FFN flops, comm[j] = rows * (w_in + d) * bytes its transfer in bytes if it
+ * runs in the Cloud (w_in = r encoded values per row, or d without a codec;
+ * plus the d-wide output row; bytes = 2 for bf16, 4 for fp32).  All output
+ * arrays hold desc->E entries; *n_tasks receives the task count.  Errors:
+ * EC2MOE_ERR_INVALID_ARG for NULL pointers, an invalid desc, or a negative
+ * count. */
+ec2moe_status ec2moe_expert_tasks(const ec2moe_layer_desc* desc, const int32_t* counts, int32_t* expert_of_task,
+                                  double* cost, double* comm, int32_t* n_tasks);
 
 /* Human-readable name of a status code (static storage). */
 const char* ec2moe_status_string(ec2moe_status status);

@@ -40,8 +40,11 @@ EXPORTED = [
     "ec2moe_lr_encode", "ec2moe_lr_decode", "ec2moe_layer_forward", "ec2moe_last_device_error",
     "ec2moe_last_launch_count", "ec2moe_status_string", "ec2moe_profile_enable", "ec2moe_profile_count",
     "ec2moe_profile_read", "ec2moe_profile_reset", "ec2moe_route_noalloc", "ec2moe_set_wait_budget",
-    "ec2moe_get_wait_budget",
+    "ec2moe_get_wait_budget", "ec2moe_schedule", "ec2moe_schedule_objective", "ec2moe_expert_tasks",
 ]
+
+END = 0
+CLOUD = 1
 
 
 class LayerDesc(ctypes.Structure):
@@ -90,6 +93,11 @@ _SIGS = {
     "ec2moe_profile_reset": (None, []),
     "ec2moe_set_wait_budget": (ctypes.c_int, [ctypes.c_int64]),
     "ec2moe_get_wait_budget": (ctypes.c_int64, []),
+    "ec2moe_schedule": (ctypes.c_int, [ctypes.c_int32, _P, _P, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                       ctypes.c_double, ctypes.c_double, _P, _P, _P, _P]),
+    "ec2moe_schedule_objective": (ctypes.c_int, [ctypes.c_int32, _P, _P, _P, ctypes.c_double, ctypes.c_double,
+                                                 ctypes.c_double, _P]),
+    "ec2moe_expert_tasks": (ctypes.c_int, [_D, _P, _P, _P, _P, _P]),
 }
 
 
@@ -263,3 +271,53 @@ def ec2moe_set_wait_budget(cycles: int) -> None:
 
 def ec2moe_get_wait_budget() -> int:
     return int(load().ec2moe_get_wait_budget())
+
+
+# ----------------------------------------------------------------- scheduler (host)
+def _dbl_array(values):
+    vals = [float(v) for v in values]
+    return (ctypes.c_double * max(1, len(vals)))(*vals), len(vals)
+
+
+def ec2moe_schedule(cost, comm, load_end=0.0, load_cloud=0.0, T_end=float("inf"), beta=0.0, eps=1e-9):
+    """Eq. 10-11 placement.  Returns (location list of END/CLOUD, visit order,
+    final End load, final Cloud load)."""
+    c, n = _dbl_array(cost)
+    m, n2 = _dbl_array(comm)
+    if n != n2:
+        raise ValueError("cost and comm differ in length")
+    loc = (ctypes.c_int32 * max(1, n))()
+    order = (ctypes.c_int32 * max(1, n))()
+    le, lc = ctypes.c_double(), ctypes.c_double()
+    _check(load().ec2moe_schedule(n, ctypes.addressof(c), ctypes.addressof(m), float(load_end), float(load_cloud),
+                                  float(T_end), float(beta), float(eps), ctypes.addressof(loc),
+                                  ctypes.addressof(order), ctypes.addressof(le), ctypes.addressof(lc)),
+           "ec2moe_schedule")
+    return list(loc)[:n], list(order)[:n], le.value, lc.value
+
+
+def ec2moe_schedule_objective(cost, comm, location, rate_end, rate_cloud, alpha) -> float:
+    """Eq. 9 objective of a placement."""
+    c, n = _dbl_array(cost)
+    m, _ = _dbl_array(comm)
+    loc = (ctypes.c_int32 * max(1, n))(*[int(v) for v in location])
+    out = ctypes.c_double()
+    _check(load().ec2moe_schedule_objective(n, ctypes.addressof(c), ctypes.addressof(m), ctypes.addressof(loc),
+                                            float(rate_end), float(rate_cloud), float(alpha),
+                                            ctypes.addressof(out)), "ec2moe_schedule_objective")
+    return out.value
+
+
+def ec2moe_expert_tasks(desc, counts):
+    """Route-aware tasks from a host histogram: (expert ids, costs, comms)."""
+    E = int(desc.E)
+    cnt = (ctypes.c_int32 * E)(*[int(v) for v in counts])
+    ids = (ctypes.c_int32 * E)()
+    cost = (ctypes.c_double * E)()
+    comm = (ctypes.c_double * E)()
+    nt = ctypes.c_int32()
+    _check(load().ec2moe_expert_tasks(_dref(desc), ctypes.addressof(cnt), ctypes.addressof(ids),
+                                      ctypes.addressof(cost), ctypes.addressof(comm), ctypes.addressof(nt)),
+           "ec2moe_expert_tasks")
+    n = nt.value
+    return list(ids)[:n], list(cost)[:n], list(comm)[:n]
