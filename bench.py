@@ -50,6 +50,9 @@ def parse():
     ap.add_argument("--workload", default="switch_bf16")
     ap.add_argument("--T", type=int, default=0, help="override the token count (0 = preset)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--pipeline", type=int, default=0,
+                    help="instead of the default line, measure the end/cloud pipelined call with this many "
+                         "micro-batches (two streams) against the same schedule on one stream")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="budget of the CPU baseline sample")
     return ap.parse_args()
 
@@ -480,10 +483,101 @@ def run_ours(args):
     return 0
 
 
+END_STAGE = ("gate_prep", "gate_topk", "lr_encode", "route", "route_count", "route_scatter")
+
+
+def run_pipeline(args):
+    """The end/cloud pipeline (ec2moe_layer_forward_pipelined) on one GPU: the
+    pipelined call on two streams, the same micro-batch schedule on one stream,
+    and the one-stream fused layer call; every step device-timed on the end
+    stream with L2 flushed in between.  Overlap efficiency = time saved by the
+    second stream / the shorter of the two stages' summed kernel times."""
+    import torch
+
+    from paper_2508_06024_gb300 import build as B
+    from paper_2508_06024_gb300 import ec2moe as C
+    from paper_2508_06024_gb300 import synth as S
+    from paper_2508_06024_gb300.runner import LayerRun
+
+    if int(os.environ.get("RANK", "0")) != 0:
+        return 0
+    B.build()
+    C.load()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    cfg = workload_config(args.workload, args.T)
+    run = LayerRun(cfg, S.make_inputs(cfg, device=dev), device=dev)
+    s_end, s_cloud = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    s_end.wait_stream(torch.cuda.current_stream(dev))
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    m = args.pipeline
+
+    def timed(fn):
+        for _ in range(max(args.warmup, 3)):
+            fn()
+        torch.cuda.synchronize(dev)
+        ts = []
+        for _ in range(args.steps):
+            with torch.cuda.stream(s_end):
+                flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s_end)
+            fn()
+            b.record(s_end)
+            torch.cuda.synchronize(dev)
+            ts.append(a.elapsed_time(b))
+        return statistics.median(ts)
+
+    t_layer = timed(lambda: run.forward(stream=s_end))
+    t_pipe = timed(lambda: run.forward_pipelined(m, s_end, s_cloud))
+    t_serial = timed(lambda: run.forward_pipelined(m, s_end, s_end))
+    status = C.ec2moe_last_device_error(s_end)
+    if status != C.OK:
+        raise RuntimeError(f"device error: {C.status_string(status)}")
+    # per-stage kernel time of the one-stream schedule
+    C.ec2moe_profile_reset()
+    C.ec2moe_profile_enable(True)
+    reps = 5
+    for _ in range(reps):
+        with torch.cuda.stream(s_end):
+            flush.zero_()
+        run.forward_pipelined(m, s_end, s_end)
+    torch.cuda.synchronize(dev)
+    end_ms = cloud_ms = 0.0
+    for i in range(C.ec2moe_profile_count()):
+        name, ms = C.ec2moe_profile_read(i)
+        if name in END_STAGE:
+            end_ms += ms
+        else:
+            cloud_ms += ms
+    C.ec2moe_profile_enable(False)
+    C.ec2moe_profile_reset()
+    end_ms /= reps
+    cloud_ms /= reps
+    line = {
+        "metric": "pipelined MoE-layer tokens/s (end stream: gate, routing, encoder; cloud stream: decoder, "
+                  "experts, combine)",
+        "value": round(cfg.T / (t_pipe * 1e-3), 1), "unit": "tokens/s", "n_gpus": 1, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(t_pipe, 5), "higher_is_better": True, "dtype":
+            "bf16" if cfg.dtype == 1 else "f32", "data": "synthetic",
+        "config": {"workload": describe(cfg), "n_micro": m, "l2": "flushed between steps (256 MiB write)",
+                   "launch": "eager C-ABI calls, device-timed on the end stream"},
+        "pipeline": {"ms_pipelined": round(t_pipe, 5), "ms_one_stream_same_schedule": round(t_serial, 5),
+                     "ms_fused_layer_call": round(t_layer, 5), "end_stage_kernel_ms": round(end_ms, 5),
+                     "cloud_stage_kernel_ms": round(cloud_ms, 5),
+                     "overlap_efficiency": round((t_serial - t_pipe) / max(min(end_ms, cloud_ms), 1e-9), 4),
+                     "speedup_vs_one_stream": round(t_serial / t_pipe, 4)},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.pipeline > 0:
+        return run_pipeline(args)
     return run_ours(args)
 
 

@@ -246,6 +246,41 @@ ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream);
 ec2moe_status ec2moe_set_wait_budget(int64_t cycles);
 int64_t ec2moe_get_wait_budget(void);
 
+/* ---------------------------------------------------------------------------
+ * The end/cloud pipeline of the paper's pipeline optimisation (PO-ECC: the end
+ * runs the gate and the low-rank encoder, the cloud the decoder and the
+ * experts, overlapped across requests), on one GPU with two CUDA streams.
+ *
+ * Same result as ec2moe_layer_forward, computed in n_micro contiguous
+ * micro-batches of ceil(T / n_micro) tokens: stream_end runs the gate, the
+ * routing and the encoder Z = X V_enc^T of micro-batch i + 1 while
+ * stream_cloud runs the decoder (rows straight into expert order), the
+ * experts, the shared experts and the combine of micro-batch i.  The
+ * micro-batch's Z and routing tables are handed from the end to the cloud
+ * through a CUDA event; counts is the sum of the micro-batches' histograms.
+ * Y, topk_idx, topk_w and Z (optional) receive every token's rows in token
+ * order, as for ec2moe_layer_forward; the order of rows inside each expert
+ * (not an output) follows the micro-batches.
+ *
+ * Streams: stream_cloud first waits for everything enqueued on stream_end
+ * before the call, and at the end stream_end waits for stream_cloud, so the
+ * call as a whole is ordered on stream_end (synchronise or capture on
+ * stream_end; stream_cloud is forked and joined inside the call).  Passing the
+ * same stream twice runs the micro-batches back to back.
+ *
+ * workspace: ec2moe_pipelined_workspace_size(desc, n_micro) bytes, 16-byte
+ * aligned; one region per micro-batch, so calls that overlap on the GPU must
+ * not share it.  1 <= n_micro <= EC2MOE_MAX_MICRO (else
+ * EC2MOE_ERR_INVALID_ARG); micro-batches beyond T tokens are empty and
+ * skipped.  Other errors as ec2moe_layer_forward. */
+#define EC2MOE_MAX_MICRO 64
+size_t ec2moe_pipelined_workspace_size(const ec2moe_layer_desc* desc, int32_t n_micro);
+ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, const ec2moe_layer_weights* w,
+                                             const void* X, const uint8_t* mask, void* Y, int32_t* topk_idx,
+                                             float* topk_w, int32_t* counts, void* Z, void* workspace,
+                                             size_t ws_bytes, int32_t n_micro, ec2moe_stream_t stream_end,
+                                             ec2moe_stream_t stream_cloud);
+
 /* Number of kernels the last successful call on this host thread enqueued. */
 int32_t ec2moe_last_launch_count(void);
 
@@ -255,7 +290,7 @@ int32_t ec2moe_last_launch_count(void);
  * stop event.  `name` receives a static string naming the launch
  * ("gate_prep", "gate_topk", "route_count", "route_scatter", "gather_rows", "lr_encode",
  * "lr_decode", "expert_up", "expert_down", "shared_up", "shared_down",
- * "combine"); `ms` its device duration.  Profiling is off by default and
+ * "combine", "sum_counts"); `ms` its device duration.  Profiling is off by default and
  * costs nothing when off. */
 ec2moe_status ec2moe_profile_enable(int32_t enable);
 int32_t ec2moe_profile_count(void);

@@ -15,6 +15,7 @@ namespace ec2moe {
 
 namespace {
 thread_local int t_launches = 0;
+thread_local bool t_plain_next = false;
 
 // Per-launch timing records (ec2moe_profile_*).  Events come from a pool that
 // is reused after ec2moe_profile_reset.
@@ -48,15 +49,19 @@ cudaEvent_t pool_event() {
 }
 }  // namespace
 
-void reset_launch_count() { t_launches = 0; }
+void reset_launch_count() {
+  t_launches = 0;
+  t_plain_next = false;
+}
 
 bool next_launch_pdl() {
   static const bool disabled = [] {
     const char* v = getenv("EC2MOE_NO_PDL");
     return v && v[0] == '1';
   }();
-  return !disabled && t_launches > 0;
+  return !disabled && t_launches > 0 && !t_plain_next;
 }
+void plain_next_launch() { t_plain_next = true; }
 int launch_count() { return t_launches; }
 
 KernelScope::KernelScope(const char* name, cudaStream_t s) : name_(name), s_(s) {
@@ -69,6 +74,7 @@ KernelScope::KernelScope(const char* name, cudaStream_t s) : name_(name), s_(s) 
 
 KernelScope::~KernelScope() {
   ++t_launches;
+  t_plain_next = false;
   std::lock_guard<std::mutex> lock(g_prof_mu);
   if (g_prof_on && start_) {
     cudaEvent_t stop = pool_event();
@@ -332,6 +338,57 @@ cudaError_t run_codec(const ec2moe_layer_desc* d, bool encode, const void* in, c
   return run_gemm(d, g, EPI_STORE, s);
 }
 
+// Argument checks of a whole-layer call (everything but the workspace).
+ec2moe_status check_layer_call(const ec2moe_layer_desc* desc, const ec2moe_layer_weights* w, const void* X,
+                               const uint8_t* mask, void* Y, int32_t* topk_idx, float* topk_w, int32_t* counts,
+                               void* Z, uint32_t mask_bits[4], bool* empty) {
+  *empty = false;
+  ec2moe_status st = check_desc(desc);
+  if (st != EC2MOE_OK) return st;
+  if (!w) return EC2MOE_ERR_INVALID_ARG;
+  st = check_mask(desc, mask, mask_bits);
+  if (st != EC2MOE_OK) return st;
+  st = check_ffn(desc, desc->d_ff);
+  if (st != EC2MOE_OK) return st;
+  if (desc->n_shared > 0) {
+    st = check_ffn(desc, desc->d_ff_shared);
+    if (st != EC2MOE_OK) return st;
+  }
+  if (desc->r > 0) {
+    st = check_codec(desc);
+    if (st != EC2MOE_OK) return st;
+  }
+  if (desc->T == 0) {
+    *empty = true;
+    return EC2MOE_OK;
+  }
+  EC2MOE_REQUIRE_PTR(X);
+  EC2MOE_REQUIRE_PTR(Y);
+  EC2MOE_REQUIRE_PTR(topk_idx);
+  EC2MOE_REQUIRE_PTR(topk_w);
+  if (!counts) return EC2MOE_ERR_INVALID_ARG;
+  EC2MOE_REQUIRE_PTR(w->W_local);
+  EC2MOE_REQUIRE_PTR(w->b_local);
+  if (desc->n_groups > 1) {
+    EC2MOE_REQUIRE_PTR(w->W_global);
+    EC2MOE_REQUIRE_PTR(w->b_global);
+  }
+  EC2MOE_REQUIRE_PTR(w->W1);
+  EC2MOE_REQUIRE_PTR(w->W2);
+  if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(w->W3);
+  if (desc->n_shared > 0) {
+    EC2MOE_REQUIRE_PTR(w->W1s);
+    EC2MOE_REQUIRE_PTR(w->W2s);
+    if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(w->W3s);
+  }
+  if (desc->r > 0) {
+    EC2MOE_REQUIRE_PTR(w->V_enc);
+    EC2MOE_REQUIRE_PTR(w->V_dec);
+    if (Z && !aligned16(Z)) return EC2MOE_ERR_MISALIGNED;
+  }
+  return EC2MOE_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -526,47 +583,10 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
                                    const uint8_t* mask, void* Y, int32_t* topk_idx, float* topk_w, int32_t* counts,
                                    void* Z, void* workspace, size_t ws_bytes, ec2moe_stream_t stream) {
   reset_launch_count();
-  ec2moe_status st = check_desc(desc);
-  if (st != EC2MOE_OK) return st;
-  if (!w) return EC2MOE_ERR_INVALID_ARG;
   GateArgs ga{};
-  st = check_mask(desc, mask, ga.mask_bits);
-  if (st != EC2MOE_OK) return st;
-  st = check_ffn(desc, desc->d_ff);
-  if (st != EC2MOE_OK) return st;
-  if (desc->n_shared > 0) {
-    st = check_ffn(desc, desc->d_ff_shared);
-    if (st != EC2MOE_OK) return st;
-  }
-  if (desc->r > 0) {
-    st = check_codec(desc);
-    if (st != EC2MOE_OK) return st;
-  }
-  if (desc->T == 0) return EC2MOE_OK;
-  EC2MOE_REQUIRE_PTR(X);
-  EC2MOE_REQUIRE_PTR(Y);
-  EC2MOE_REQUIRE_PTR(topk_idx);
-  EC2MOE_REQUIRE_PTR(topk_w);
-  if (!counts) return EC2MOE_ERR_INVALID_ARG;
-  EC2MOE_REQUIRE_PTR(w->W_local);
-  EC2MOE_REQUIRE_PTR(w->b_local);
-  if (desc->n_groups > 1) {
-    EC2MOE_REQUIRE_PTR(w->W_global);
-    EC2MOE_REQUIRE_PTR(w->b_global);
-  }
-  EC2MOE_REQUIRE_PTR(w->W1);
-  EC2MOE_REQUIRE_PTR(w->W2);
-  if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(w->W3);
-  if (desc->n_shared > 0) {
-    EC2MOE_REQUIRE_PTR(w->W1s);
-    EC2MOE_REQUIRE_PTR(w->W2s);
-    if (desc->act == EC2MOE_SWIGLU) EC2MOE_REQUIRE_PTR(w->W3s);
-  }
-  if (desc->r > 0) {
-    EC2MOE_REQUIRE_PTR(w->V_enc);
-    EC2MOE_REQUIRE_PTR(w->V_dec);
-    if (Z && !aligned16(Z)) return EC2MOE_ERR_MISALIGNED;
-  }
+  bool empty = false;
+  ec2moe_status st = check_layer_call(desc, w, X, mask, Y, topk_idx, topk_w, counts, Z, ga.mask_bits, &empty);
+  if (st != EC2MOE_OK || empty) return st;
   const LayerWs L = layer_ws(desc);
   if (!workspace || ws_bytes < L.total) return EC2MOE_ERR_WORKSPACE;
   if (!aligned16(workspace)) return EC2MOE_ERR_MISALIGNED;
@@ -576,8 +596,7 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   const size_t es = esize(desc);
   const long long T = desc->T, k = desc->k, n = T * k;
   void* zbuf = (desc->r > 0) ? (Z ? Z : ws + L.z) : nullptr;
-  uint8_t* xa = ws + L.xa;                      // [n + T, d]
-  uint8_t* x_hat = xa + (size_t)n * desc->d * es;  // rows [n, n + T)
+  uint8_t* xa = ws + L.xa;  // [n + T, d]: expert-ordered rows, then X_hat
   void* h = ws + L.h;
   const bool direct = (k == 1 && desc->n_shared == 0);
   void* slot = direct ? Y : static_cast<void*>(ws + L.slot);
@@ -659,7 +678,6 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
     shared_a_rows = T;
     shared_a_base = 0;
   }
-  (void)x_hat;
   // Steps 4-5a: routed experts, gate scale and unpermute fused in the down projection.
   int n_allowed = 0;
   for (int e = 0; e < desc->E; ++e) n_allowed += mask[e] ? 1 : 0;
@@ -672,6 +690,147 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   }
   // Step 5b: fixed-order combine (skipped when the down projection wrote Y directly).
   if (!direct) EC2MOE_CUDA(launch_combine(slot, shared, desc->n_shared, Y, desc->T, desc->k, desc->d, bf, stream));
+  return EC2MOE_OK;
+}
+
+size_t ec2moe_pipelined_workspace_size(const ec2moe_layer_desc* desc, int32_t n_micro) {
+  if (check_desc(desc) != EC2MOE_OK || n_micro < 1 || n_micro > EC2MOE_MAX_MICRO) return 0;
+  ec2moe_layer_desc sub = *desc;
+  sub.T = (desc->T + n_micro - 1) / n_micro;
+  return (size_t)n_micro * align_up(layer_ws(&sub).total) + align_up((size_t)n_micro * desc->E * 4);
+}
+
+// The end/cloud pipeline of the paper's PO-ECC stage on one GPU: the tokens
+// are cut into n_micro contiguous micro-batches; the end stream runs the gate,
+// the routing and the encoder (Z) of micro-batch i + 1 while the cloud stream
+// runs the decoder, the experts and the combine of micro-batch i.  Each
+// micro-batch has its own workspace region, so the two streams share only the
+// events that hand Z (and the routing tables) from the end to the cloud.
+ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, const ec2moe_layer_weights* w,
+                                             const void* X, const uint8_t* mask, void* Y, int32_t* topk_idx,
+                                             float* topk_w, int32_t* counts, void* Z, void* workspace,
+                                             size_t ws_bytes, int32_t n_micro, ec2moe_stream_t stream_end,
+                                             ec2moe_stream_t stream_cloud) {
+  reset_launch_count();
+  GateArgs ga0{};
+  bool empty = false;
+  ec2moe_status st = check_layer_call(desc, w, X, mask, Y, topk_idx, topk_w, counts, Z, ga0.mask_bits, &empty);
+  if (st != EC2MOE_OK || empty) return st;
+  if (n_micro < 1 || n_micro > EC2MOE_MAX_MICRO) return EC2MOE_ERR_INVALID_ARG;
+  const size_t need = ec2moe_pipelined_workspace_size(desc, n_micro);
+  if (!workspace || need == 0 || ws_bytes < need) return EC2MOE_ERR_WORKSPACE;
+  if (!aligned16(workspace)) return EC2MOE_ERR_MISALIGNED;
+
+  const bool bf = is_bf16(desc);
+  const size_t es = esize(desc);
+  const int Tm = (desc->T + n_micro - 1) / n_micro;
+  ec2moe_layer_desc full_sub = *desc;
+  full_sub.T = Tm;
+  const size_t region = align_up(layer_ws(&full_sub).total);
+  uint8_t* base = static_cast<uint8_t*>(workspace);
+  int32_t* parts = reinterpret_cast<int32_t*>(base + (size_t)n_micro * region);
+  int n_allowed = 0;
+  for (int e = 0; e < desc->E; ++e) n_allowed += mask[e] ? 1 : 0;
+
+  // one event per micro-batch hand-off, plus the fork and the join
+  thread_local std::vector<cudaEvent_t> events;
+  while ((int)events.size() < n_micro + 2) {
+    cudaEvent_t e = nullptr;
+    EC2MOE_CUDA(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+    events.push_back(e);
+  }
+  cudaStream_t se = stream_end, sc = stream_cloud;
+  EC2MOE_CUDA(cudaEventRecord(events[0], se));
+  EC2MOE_CUDA(cudaStreamWaitEvent(sc, events[0], 0));
+
+  int used = 0;
+  for (int i = 0; i < n_micro; ++i) {
+    const long long t0 = (long long)i * Tm;
+    if (t0 >= desc->T) break;
+    ++used;
+    ec2moe_layer_desc sub = *desc;
+    sub.T = (int)((desc->T - t0) < Tm ? (desc->T - t0) : Tm);
+    const LayerWs L = layer_ws(&sub);
+    uint8_t* ws = base + (size_t)i * region;
+    const long long T = sub.T, k = sub.k, n = T * k;
+    const void* Xi = static_cast<const uint8_t*>(X) + (size_t)t0 * sub.d * es;
+    void* Yi = static_cast<uint8_t*>(Y) + (size_t)t0 * sub.d * es;
+    int32_t* idx_i = topk_idx + t0 * k;
+    float* tw_i = topk_w + t0 * k;
+    int32_t* cnt_i = parts + (size_t)i * desc->E;
+    void* zbuf = (sub.r > 0) ? (Z ? static_cast<void*>(static_cast<uint8_t*>(Z) + (size_t)t0 * sub.r * es)
+                                  : static_cast<void*>(ws + L.z))
+                             : nullptr;
+    uint8_t* xa = ws + L.xa;
+    void* h = ws + L.h;
+    const bool direct = (k == 1 && sub.n_shared == 0);
+    void* slot = direct ? Yi : static_cast<void*>(ws + L.slot);
+    void* shared = sub.n_shared > 0 ? static_cast<void*>(ws + L.shared) : nullptr;
+    int32_t* perm = reinterpret_cast<int32_t*>(ws + L.perm);
+    int32_t* inv_perm = reinterpret_cast<int32_t*>(ws + L.inv_perm);
+    int32_t* offsets = reinterpret_cast<int32_t*>(ws + L.offsets);
+    int32_t* blk = reinterpret_cast<int32_t*>(ws + L.blk);
+
+    // ---- end: gate, routing, encoder
+    GateArgs ga = ga0;
+    ga.X = Xi;
+    ga.W_local = w->W_local;
+    ga.b_local = w->b_local;
+    ga.W_global = sub.n_groups > 1 ? w->W_global : nullptr;
+    ga.b_global = sub.n_groups > 1 ? w->b_global : nullptr;
+    ga.T = sub.T;
+    ga.d = sub.d;
+    ga.E = sub.E;
+    ga.K = sub.n_groups;
+    ga.k = sub.k;
+    ga.renorm = sub.renorm_topk;
+    ga.topk_idx = idx_i;
+    ga.topk_w = tw_i;
+    if (bf) {
+      ga.route_counts = cnt_i;
+      ga.route_rel = inv_perm;
+      if (gate_split_bytes(sub.E, sub.n_groups, sub.d, bf)) ga.w_split = ws + L.wsplit;
+    }
+    bool routed = false;
+    EC2MOE_CUDA(launch_gate(ga, bf, se, &routed));
+    if (!routed) EC2MOE_CUDA(launch_route(idx_i, n, sub.E, blk, cnt_i, offsets, perm, inv_perm, se));
+    if (sub.r > 0) EC2MOE_CUDA(run_codec(&sub, true, Xi, w->V_enc, zbuf, se));
+    EC2MOE_CUDA(cudaEventRecord(events[1 + i], se));
+
+    // ---- cloud: decoder into expert order, experts, combine
+    EC2MOE_CUDA(cudaStreamWaitEvent(sc, events[1 + i], 0));
+    plain_next_launch();
+    RelPlace rel;
+    if (routed) {
+      rel.counts = cnt_i;
+      rel.idx = idx_i;
+      rel.perm_out = perm;
+      rel.offsets_out = offsets;
+    }
+    const void* shared_a = xa;
+    long long shared_a_rows = n + T, shared_a_base = n;
+    if (sub.r > 0) {
+      EC2MOE_CUDA(run_codec(&sub, false, zbuf, w->V_dec, xa, sc, inv_perm, sub.n_shared > 0 ? n : -1, rel));
+    } else {
+      if (routed)
+        EC2MOE_CUDA(launch_gather_rel(Xi, xa, idx_i, cnt_i, inv_perm, perm, offsets, sub.E, n, sub.k, sub.d, bf, sc));
+      else
+        EC2MOE_CUDA(launch_gather(Xi, xa, perm, n, sub.k, sub.d, bf, sc));
+      shared_a = Xi;
+      shared_a_rows = T;
+      shared_a_base = 0;
+    }
+    EC2MOE_CUDA(run_ffn(&sub, true, xa, n + T, 0, offsets, w->W1, w->W3, w->W2, h, n + (long long)sub.n_shared * T, 0,
+                        perm, tw_i, slot, 0, sc, n_allowed));
+    if (sub.n_shared > 0)
+      EC2MOE_CUDA(run_ffn(&sub, false, shared_a, shared_a_rows, shared_a_base, nullptr, w->W1s, w->W3s, w->W2s, h,
+                          n + (long long)sub.n_shared * T, n, nullptr, nullptr, shared, 0, sc));
+    if (!direct) EC2MOE_CUDA(launch_combine(slot, shared, sub.n_shared, Yi, sub.T, sub.k, sub.d, bf, sc));
+  }
+  // the layer's histogram is the sum of the micro-batches' ones
+  EC2MOE_CUDA(launch_sum_counts(parts, used, desc->E, counts, sc));
+  EC2MOE_CUDA(cudaEventRecord(events[n_micro + 1], sc));
+  EC2MOE_CUDA(cudaStreamWaitEvent(se, events[n_micro + 1], 0));
   return EC2MOE_OK;
 }
 

@@ -37,6 +37,9 @@ int sm_count();
 // raced.  Kernels only read data produced earlier in the stream after
 // griddepcontrol.wait.
 bool next_launch_pdl();
+// Makes the next launch of the current call a plain one (full stream
+// ordering), e.g. the first kernel on a stream after a cross-stream wait.
+void plain_next_launch();
 
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_kernel(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
@@ -107,6 +110,8 @@ cudaError_t launch_route_noalloc(const int32_t* topk_idx, long long n_entries, i
 // dst[p] = src[perm[p] / k] for p < rows, width elements per row.
 cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long long rows, int k, int width,
                           bool bf16, cudaStream_t s);
+// counts[e] = sum_p parts[p*E + e], p ascending.
+cudaError_t launch_sum_counts(const int32_t* parts, int n_parts, int E, int32_t* counts, cudaStream_t s);
 // y[t] = sum_s slot[t*k+s] + sum_j shared[j*T+t]
 cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d,
                            bool bf16, cudaStream_t s);

@@ -356,6 +356,23 @@ cudaError_t launch_gather_rel(const void* src, void* dst, const int32_t* topk_id
                        offsets, E, n, k, row_bytes);
 }
 
+__global__ void sum_counts_kernel(const int32_t* __restrict__ parts, int n_parts, int E, int32_t* __restrict__ counts) {
+  pdl_trigger();
+  pdl_wait();
+  for (int e = blockIdx.x * blockDim.x + threadIdx.x; e < E; e += gridDim.x * blockDim.x) {
+    int32_t c = 0;
+    for (int p = 0; p < n_parts; ++p) c += parts[(size_t)p * E + e];
+    counts[e] = c;
+  }
+}
+
+cudaError_t launch_sum_counts(const int32_t* parts, int n_parts, int E, int32_t* counts, cudaStream_t s) {
+  KernelScope ks("sum_counts", s);
+  cudaError_t e = launch_kernel(sum_counts_kernel, dim3(1), dim3(128), 0, s, parts, n_parts, E, counts);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
 cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d, bool bf16,
                            cudaStream_t s) {
   if (T <= 0) return cudaSuccess;

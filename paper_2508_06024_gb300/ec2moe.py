@@ -41,6 +41,7 @@ EXPORTED = [
     "ec2moe_last_launch_count", "ec2moe_status_string", "ec2moe_profile_enable", "ec2moe_profile_count",
     "ec2moe_profile_read", "ec2moe_profile_reset", "ec2moe_route_noalloc", "ec2moe_set_wait_budget",
     "ec2moe_get_wait_budget", "ec2moe_schedule", "ec2moe_schedule_objective", "ec2moe_expert_tasks",
+    "ec2moe_pipelined_workspace_size", "ec2moe_layer_forward_pipelined",
 ]
 
 END = 0
@@ -98,6 +99,9 @@ _SIGS = {
     "ec2moe_schedule_objective": (ctypes.c_int, [ctypes.c_int32, _P, _P, _P, ctypes.c_double, ctypes.c_double,
                                                  ctypes.c_double, _P]),
     "ec2moe_expert_tasks": (ctypes.c_int, [_D, _P, _P, _P, _P, _P]),
+    "ec2moe_pipelined_workspace_size": (ctypes.c_size_t, [_D, ctypes.c_int32]),
+    "ec2moe_layer_forward_pipelined": (ctypes.c_int, [_D, ctypes.POINTER(LayerWeights), _P, _P, _P, _P, _P, _P, _P,
+                                                      _P, ctypes.c_size_t, ctypes.c_int32, _P, _P]),
 }
 
 
@@ -235,6 +239,18 @@ def ec2moe_layer_forward(desc, weights: LayerWeights, X, mask, Y, topk_idx, topk
     _check(load().ec2moe_layer_forward(_dref(desc), ctypes.byref(weights), _ptr(X), _mask(mask), _ptr(Y),
                                        _ptr(topk_idx), _ptr(topk_w), _ptr(counts), _ptr(Z), _ptr(workspace),
                                        int(ws_bytes), _stream(stream)), "ec2moe_layer_forward")
+
+
+def ec2moe_pipelined_workspace_size(desc: LayerDesc, n_micro: int) -> int:
+    return int(load().ec2moe_pipelined_workspace_size(_dref(desc), int(n_micro)))
+
+
+def ec2moe_layer_forward_pipelined(desc, weights: LayerWeights, X, mask, Y, topk_idx, topk_w, counts, Z, workspace,
+                                   ws_bytes, n_micro, stream_end=None, stream_cloud=None):
+    _check(load().ec2moe_layer_forward_pipelined(_dref(desc), ctypes.byref(weights), _ptr(X), _mask(mask), _ptr(Y),
+                                                 _ptr(topk_idx), _ptr(topk_w), _ptr(counts), _ptr(Z),
+                                                 _ptr(workspace), int(ws_bytes), int(n_micro), _stream(stream_end),
+                                                 _stream(stream_cloud)), "ec2moe_layer_forward_pipelined")
 
 
 def ec2moe_last_device_error(stream=None) -> int:

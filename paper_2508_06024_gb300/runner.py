@@ -46,6 +46,17 @@ class LayerRun:
         self.ws_bytes = C.ec2moe_workspace_size(self.desc)
         self.workspace = torch.empty(max(self.ws_bytes, 16), dtype=torch.uint8, device=device)
 
+    def forward_pipelined(self, n_micro: int, stream_end=None, stream_cloud=None,
+                          X: Optional[torch.Tensor] = None) -> torch.Tensor:
+        """The end/cloud pipelined layer call (two streams, n_micro micro-batches)."""
+        need = C.ec2moe_pipelined_workspace_size(self.desc, n_micro)
+        if getattr(self, "pws", None) is None or self.pws.numel() < need:
+            self.pws = torch.empty(max(need, 16), dtype=torch.uint8, device=self.Y.device)
+        C.ec2moe_layer_forward_pipelined(self.desc, self.weights, self.inp["X"] if X is None else X, self.mask,
+                                         self.Y, self.topk_idx, self.topk_w, self.counts, self.Z, self.pws,
+                                         self.pws.numel(), n_micro, stream_end, stream_cloud)
+        return self.Y
+
     def forward(self, X: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
         C.ec2moe_layer_forward(self.desc, self.weights, self.inp["X"] if X is None else X, self.mask, self.Y,
                                self.topk_idx, self.topk_w, self.counts, self.Z, self.workspace, self.ws_bytes,

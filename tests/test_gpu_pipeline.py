@@ -1,0 +1,94 @@
+"""The end/cloud pipelined layer call (two streams, micro-batches) through the
+C ABI: same routing, histogram, transmitted Z and output as the one-stream
+layer call, and parity with the oracle."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import ec2moe_oracle as orc
+from paper_2508_06024_gb300 import build as B
+from paper_2508_06024_gb300 import ec2moe as C
+from paper_2508_06024_gb300 import synth as S
+from paper_2508_06024_gb300.runner import LayerRun
+from tests.parity import TIE_GAP, oracle_inputs, output_check, routing_check
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    B.build()
+    C.load()
+    yield
+    torch.cuda.synchronize()
+
+
+def _pipelined(run, n_micro, same_stream=False):
+    cur = torch.cuda.current_stream()
+    s_end = torch.cuda.Stream()
+    s_cloud = s_end if same_stream else torch.cuda.Stream()
+    s_end.wait_stream(cur)
+    run.Y.fill_(float("nan"))
+    run.topk_idx.fill_(-1)
+    run.counts.fill_(-1)
+    run.forward_pipelined(n_micro, s_end, s_cloud)
+    cur.wait_stream(s_end)
+    torch.cuda.synchronize()
+    assert C.ec2moe_last_device_error() == C.OK
+    return (run.Y.clone(), run.topk_idx.clone(), run.topk_w.clone(), run.counts.clone(),
+            None if run.Z is None else run.Z.clone())
+
+
+PIPE_CASES = [
+    (S.preset("switch_bf16", T=1000, seed=31), 3),
+    (S.preset("switch_bf16", T=1000, k=2, n_groups=4, seed=37), 5),
+    (S.preset("finegrained_bf16", T=777, seed=32), 4),
+    (S.preset("mixtral_bf16", T=600, seed=35), 2),
+    (S.preset("switch_bf16", T=300, r=0, seed=34), 2),
+    (S.preset("tiny_fp32", seed=33), 2),
+    (S.preset("decode_bf16", T=5, n_allowed=8, seed=36), 8),
+    (S.preset("switch_bf16", T=4096), 1),
+]
+
+
+@pytest.mark.parametrize("cfg,n_micro", PIPE_CASES,
+                         ids=lambda v: f"{v.name}-T{v.T}-k{v.k}-r{v.r}" if hasattr(v, "name") else f"m{v}")
+def test_pipelined_matches_one_stream_layer(cfg, n_micro):
+    inp = S.make_inputs(cfg, device="cuda")
+    run = LayerRun(cfg, inp)
+    run.forward()
+    torch.cuda.synchronize()
+    ref = (run.Y.clone(), run.topk_idx.clone(), run.topk_w.clone(), run.counts.clone(),
+           None if run.Z is None else run.Z.clone())
+    for same in (False, True):
+        got = _pipelined(run, n_micro, same_stream=same)
+        assert torch.equal(got[1], ref[1]) and torch.equal(got[2], ref[2]) and torch.equal(got[3], ref[3])
+        if ref[4] is not None:
+            assert torch.equal(got[4], ref[4])
+        assert torch.equal(got[0], ref[0])
+
+
+def test_pipelined_parity_with_oracle():
+    cfg = S.preset("finegrained_bf16", T=513, seed=38)
+    inp = S.make_inputs(cfg, device="cuda")
+    run = LayerRun(cfg, inp)
+    Y, idx, w, counts, Z = _pipelined(run, 3)
+    o = oracle_inputs(inp, lazy_experts=True)
+    ref = orc.layer_forward(o, cfg.n_groups, cfg.k, cfg.act, bool(cfg.renorm_topk))
+    gi = idx.cpu().numpy()
+    routing_check(gi, ref)
+    keep = ref["gap_boundary"] >= TIE_GAP
+    assert np.array_equal(counts.cpu().numpy(), np.bincount(gi.ravel(), minlength=cfg.E))
+    y = Y.detach().to("cpu", torch.float64).numpy()
+    output_check(y[keep], ref["y"][keep], True)
+    output_check(Z.detach().to("cpu", torch.float64).numpy(), ref["Z"], True)
+
+
+def test_pipelined_rejects_bad_micro_count():
+    cfg = S.preset("switch_bf16", T=256, seed=39)
+    run = LayerRun(cfg, S.make_inputs(cfg, device="cuda"))
+    for bad in (0, C.load() and 65):
+        with pytest.raises(C.Ec2moeError):
+            C.ec2moe_layer_forward_pipelined(run.desc, run.weights, run.inp["X"], run.mask, run.Y, run.topk_idx,
+                                             run.topk_w, run.counts, run.Z, run.workspace, run.ws_bytes, bad)
+    assert C.ec2moe_pipelined_workspace_size(run.desc, 0) == 0
