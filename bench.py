@@ -109,7 +109,10 @@ def kernel_work(cfg, name: str):
     if name == "lr_encode":
         return 2.0 * T * d * r, es * (T * d + r * d + T * r)
     if name == "lr_decode":
-        return 2.0 * T * r * d, es * (T * r + d * r + T * d)
+        # layer path: each decoded row is written to its k expert-order slots
+        # (plus the shared experts' copy)
+        rows_out = n + (T if cfg.n_shared > 0 else 0)
+        return 2.0 * T * r * d, es * (T * r + d * r + rows_out * d)
     if name == "lr_codec":
         return 4.0 * T * d * r, es * (T * d + 2 * r * d + T * r + n * d)
     if name == "gate_topk":

@@ -418,7 +418,10 @@ cudaError_t launch_r(const CodecArgs& a, cudaStream_t s) {
 
 }  // namespace
 
-bool codec_fused_supported(int d, int r) { return (r == 128 || r == 256) && d % 64 == 0 && d >= 128; }
+// Every CTA of a token tile recomputes Z (reading the tile's X rows and all of
+// V_enc), so the fused kernel pays off only while a tile has few d-chunks: up
+// to d = 1024 (four chunks of 256).  Wider layers run the two GEMMs apart.
+bool codec_fused_supported(int d, int r) { return (r == 128 || r == 256) && d % 64 == 0 && d >= 128 && d <= 1024; }
 
 cudaError_t launch_codec_fused(const CodecArgs& a, cudaStream_t s) {
   if (!codec_fused_supported(a.d, a.r) || a.k < 1 || a.k > 8 || a.E > 128) return cudaErrorInvalidValue;
