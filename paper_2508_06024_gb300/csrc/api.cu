@@ -235,7 +235,10 @@ GemmArgs gemm_base() {
 }
 
 cudaError_t run_gemm(const ec2moe_layer_desc* d, const GemmArgs& g, int epi, cudaStream_t s) {
-  return is_bf16(d) ? launch_gemm_tc(g, epi, s) : launch_gemm_simt(g, epi, s);
+  if (!is_bf16(d)) return launch_gemm_simt(g, epi, s);
+  // decode-sized groups: stream each weight row once on the CUDA cores
+  if (gemm_skinny_supported(g, epi)) return launch_gemm_skinny(g, epi, s);
+  return launch_gemm_tc(g, epi, s);
 }
 
 // Up projection (+ activation) then down projection over groups of rows.
@@ -269,6 +272,7 @@ cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long
   up.out = H;
   up.ldo = ff;
   up.max_rows = rows;
+  up.group_rows_bound = routed ? rows : d->T;
   up.g_active = routed ? g_active : 0;
   cudaError_t e = run_gemm(d, up, act_epi, s);
   if (e != cudaSuccess) return e;
@@ -293,6 +297,7 @@ cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long
   dn.perm = routed ? perm : nullptr;
   dn.scale = routed ? scale : nullptr;
   dn.max_rows = rows;
+  dn.group_rows_bound = routed ? rows : d->T;
   dn.g_active = routed ? g_active : 0;
   return run_gemm(d, dn, routed ? EPI_SCATTER : EPI_STORE, s);
 }

@@ -149,11 +149,16 @@ struct GemmArgs {
   int rep_E;
   long long max_rows;                // upper bound of sum_g M_g (for the grid size)
   int g_active;                      // groups expected to hold rows (tile-count estimate; 0 = G)
+  long long group_rows_bound;        // upper bound of every M_g known on the host (0 = none)
   long long timeout_cycles;          // bounded-wait budget (tensor-core path)
   const char* name;                  // label for per-launch profiling (nullptr = by epilogue)
 };
 cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s);    // bf16, tcgen05
 cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s);  // fp32, CUDA cores
+// bf16 groups of at most 16 rows (decode batches): weight rows streamed once
+// on the CUDA cores; every epilogue but EPI_REPLICATE.
+bool gemm_skinny_supported(const GemmArgs& a, int epi);
+cudaError_t launch_gemm_skinny(const GemmArgs& a, int epi, cudaStream_t s);
 // 2-D bf16 tensor map over a row-major [rows, cols] matrix: box 64 columns x
 // box_rows rows, 128-byte swizzle, zero fill out of bounds (cached).
 bool make_tensor_map_bf16(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows);

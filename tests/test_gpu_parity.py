@@ -189,6 +189,13 @@ LAYER_CASES = [
     (S.preset("decode_bf16", T=1, n_allowed=4, r=128, seed=1), None),
     (S.preset("decode_bf16", T=16, n_allowed=8, r=256, seed=16), None),
     (S.preset("decode_bf16", T=256, n_allowed=4, r=512, seed=256), None),
+    # decode-sized groups (the weight-streaming CUDA-core GEMM at <= 2 rows)
+    (S.preset("decode_bf16", T=4, n_allowed=8, r=256, seed=41), None),
+    (S.preset("finegrained_bf16", T=2, seed=42), None),
+    (S.preset("switch_bf16", T=2, seed=43), None),
+    (S.preset("decode_bf16", T=1, n_allowed=8, r=256, seed=46), None),
+    (S.preset("mixtral_bf16", T=3, seed=44), None),
+    (S.preset("tiny_fp32", T=7, seed=45), None),
 ]
 
 

@@ -65,7 +65,13 @@ def test_pipelined_matches_one_stream_layer(cfg, n_micro):
         assert torch.equal(got[1], ref[1]) and torch.equal(got[2], ref[2]) and torch.equal(got[3], ref[3])
         if ref[4] is not None:
             assert torch.equal(got[4], ref[4])
-        assert torch.equal(got[0], ref[0])
+        if cfg.T * cfg.k <= 2 or -(-cfg.T // n_micro) * cfg.k > 2:
+            assert torch.equal(got[0], ref[0])  # the same GEMM path on both sides
+        else:
+            # micro-batches of <= 2 rows per expert take the weight-streaming
+            # GEMM, the whole batch the tensor-core one: equal up to rounding
+            output_check(got[0].to("cpu", torch.float64).numpy(), ref[0].to("cpu", torch.float64).numpy(),
+                         cfg.dtype == S.BF16)
 
 
 def test_pipelined_parity_with_oracle():
