@@ -1,4 +1,4 @@
-// Grouped bf16 GEMM for groups of at most SK_MAXR rows (decode-sized expert
+// Grouped bf16 GEMM for groups of at most 16 rows (decode-sized expert
 // batches, Eq. 1 steps 4-5): C_g = A_g B_g^T where every group holds only a
 // few token rows, so the work is streaming the weight rows once.
 //
@@ -25,7 +25,6 @@ constexpr int SK_WARPS = 8;
 constexpr int SK_THREADS = 32 * SK_WARPS;
 constexpr int SK_CPW = 2;     // output columns per warp
 constexpr int SK_KC = 1024;   // K columns per staged chunk (four 16-byte pieces per lane)
-constexpr int SK_MAXR = 16;   // rows per group (at most)
 
 struct SkParams {
   const __nv_bfloat16* A;
