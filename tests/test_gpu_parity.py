@@ -196,6 +196,10 @@ LAYER_CASES = [
     (S.preset("decode_bf16", T=1, n_allowed=8, r=256, seed=46), None),
     (S.preset("mixtral_bf16", T=3, seed=44), None),
     (S.preset("tiny_fp32", T=7, seed=45), None),
+    # the limits: 128 experts in 16 groups, Top-8, 144 gate rows; and many
+    # tiles per CTA in every kernel
+    (S.preset("switch_bf16", T=1024, d=512, E=128, d_ff=512, n_groups=16, k=8, n_allowed=96, r=128, seed=47), 256),
+    (S.preset("switch_bf16", T=65536, seed=48), 256),
 ]
 
 
