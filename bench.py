@@ -84,17 +84,18 @@ def load_peaks():
 
 
 # ------------------------------------------------------------------ algorithmic work per launch
-def kernel_work(cfg, name: str):
+def kernel_work(cfg, name: str, touched: int = 0):
     """(flops, bytes) of one launch of a named kernel, from the layer shape.
 
-    GEMM bytes count the weights of the allowed experts once plus activations
-    read and written once; gate bytes count X, the gate weights and the Top-k
-    outputs; data-movement kernels count each row read and written once.
+    GEMM bytes count the weights of the experts that received rows (`touched`;
+    0 = every allowed expert) once plus activations read and written once;
+    gate bytes count X, the gate weights and the Top-k outputs; data-movement
+    kernels count each row read and written once.
     """
     es = 2 if cfg.dtype == 1 else 4
     T, d, k, E, r, ff = cfg.T, cfg.d, cfg.k, cfg.E, cfg.r, cfg.d_ff
     n = T * k
-    na = cfg.n_allowed
+    na = touched if touched > 0 else cfg.n_allowed
     glu = 2 if cfg.act == 1 else 1
     K = cfg.n_groups if cfg.n_groups > 1 else 0
     if name == "expert_up":
@@ -129,11 +130,14 @@ def kernel_work(cfg, name: str):
     return 0.0, 0.0
 
 
-def roofline_for(cfg, name, avg_ms, peaks, peaks_src, traffic):
-    flops, byts = kernel_work(cfg, name)
+def roofline_for(cfg, name, avg_ms, peaks, peaks_src, traffic, touched: int = 0):
+    """The kernel's roofline: tensor when its arithmetic intensity is at or
+    above the ridge of the measured peaks (GEMMs of large batches), else HBM
+    (data movement, the gate, decode-sized GEMMs that stream their weights)."""
+    flops, byts = kernel_work(cfg, name, touched)
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
-    tensor = name in ("expert_up", "expert_down", "shared_up", "shared_down") or (
-        name in ("lr_encode", "lr_decode") and flops / max(byts, 1) >= ridge)
+    tensor = name in ("expert_up", "expert_down", "shared_up", "shared_down", "lr_encode", "lr_decode") and (
+        flops / max(byts, 1) >= ridge)
     sec = avg_ms * 1e-3
     if tensor and cfg.dtype == 1:
         achieved = flops / sec / 1e12
@@ -446,9 +450,10 @@ def run_ours(args):
         k["share"] = round(k["avg_ms"] * k["launches_per_step"] / tot, 4) if tot else 0.0
         k["avg_ms"] = round(k["avg_ms"], 5)
     dominant = max(kern, key=lambda n: kern[n]["avg_ms"] * kern[n]["launches_per_step"])
+    touched = int((run.counts > 0).sum().item())
     roof = roofline_for(cfg, dominant, kern[dominant]["avg_ms"], peaks, peaks_src,
-                        committed_traffic(cfg, dominant))
-    others = {n: roofline_for(cfg, n, kern[n]["avg_ms"], peaks, peaks_src, committed_traffic(cfg, n))
+                        committed_traffic(cfg, dominant), touched)
+    others = {n: roofline_for(cfg, n, kern[n]["avg_ms"], peaks, peaks_src, committed_traffic(cfg, n), touched)
               for n in kern}
     layer_flops = sum(kernel_work(cfg, n)[0] * kern[n]["launches_per_step"] for n in kern)
 
