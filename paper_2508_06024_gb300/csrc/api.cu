@@ -198,8 +198,41 @@ ec2moe_status check_mask(const ec2moe_layer_desc* d, const uint8_t* mask, uint32
   } while (0)
 
 // Workspace of ec2moe_layer_forward, each region 256-byte aligned.
+// Split-K of the routed down projection for decode-sized batches: with few
+// rows per expert only (experts with rows) x (d / 256) output tiles exist for
+// a long K = d_ff, fewer than the SMs, each streaming its weights alone; the
+// K range is split so every SM streams, the partial sums (fp32) are reduced,
+// weighted and combined by one small kernel.
+constexpr int SPLITK_MAX = 8;
+bool splitk_possible(const ec2moe_layer_desc* d) {
+  const long long n = (long long)d->T * d->k;
+  return d->dtype == EC2MOE_BF16 && n > 4 && n <= 128 && d->d_ff >= 4096 && d->d % 4 == 0;
+}
+// The split whose (tile x K range) units fill whole waves of the SMs best
+// (expected m-tiles: one per expert with rows, at least n / 128).
+int splitk_factor(const ec2moe_layer_desc* d, int n_allowed) {
+  if (!splitk_possible(d)) return 1;
+  const long long n = (long long)d->T * d->k;
+  const long long experts = n < n_allowed ? n : n_allowed;
+  const long long m_tiles = experts > (n + 127) / 128 ? experts : (n + 127) / 128;
+  const long long tiles = m_tiles * ((d->d + 255) / 256);
+  const long long sms = sm_count();
+  int best = 1;
+  double best_eff = -1.0;
+  for (int sp = 1; sp <= SPLITK_MAX; ++sp) {
+    const long long units = tiles * sp;
+    const long long waves = (units + sms - 1) / sms;
+    const double eff = (double)units / (double)(waves * sms) - 0.002 * sp;  // prefer fewer splits on ties
+    if (eff > best_eff) {
+      best_eff = eff;
+      best = sp;
+    }
+  }
+  return best;
+}
+
 struct LayerWs {
-  size_t z, xa, h, slot, shared, perm, inv_perm, offsets, blk, wsplit, total;
+  size_t z, xa, h, slot, shared, perm, inv_perm, offsets, blk, wsplit, part, total;
 };
 LayerWs layer_ws(const ec2moe_layer_desc* d) {
   LayerWs w{};
@@ -223,6 +256,7 @@ LayerWs layer_ws(const ec2moe_layer_desc* d) {
   w.offsets = take((d->E + 1) * 4);
   w.blk = take((size_t)route_blocks((long long)T * k) * d->E * 4);
   w.wsplit = take(gate_split_bytes(d->E, d->n_groups, d->d, is_bf16(d)));
+  w.part = take(splitk_possible(d) ? (size_t)SPLITK_MAX * T * k * dm * 4 : 0);
   w.total = off;
   return w;
 }
@@ -248,7 +282,7 @@ cudaError_t run_gemm(const ec2moe_layer_desc* d, const GemmArgs& g, int epi, cud
 cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long long a_rows, long long a_row_base,
                     const int32_t* offsets, const void* W1, const void* W3, const void* W2, void* H, long long h_rows,
                     long long h_row_base, const int32_t* perm, const float* scale, void* out, long long out_row_base,
-                    cudaStream_t s, int g_active = 0) {
+                    cudaStream_t s, int g_active = 0, float* partial = nullptr, int split_k = 1) {
   const int ff = routed ? d->d_ff : d->d_ff_shared;
   const int G = routed ? d->E : d->n_shared;
   const long long rows = routed ? (long long)d->T * d->k : (long long)d->T * d->n_shared;
@@ -296,6 +330,15 @@ cudaError_t run_ffn(const ec2moe_layer_desc* d, bool routed, const void* A, long
   dn.ldo = d->d;
   dn.perm = routed ? perm : nullptr;
   dn.scale = routed ? scale : nullptr;
+  if (routed && split_k > 1 && partial) {
+    // split-K partial sums; the gate weights and the unpermute come in the reduce
+    dn.split_k = split_k;
+    dn.partial = partial;
+    dn.part_rows = rows;
+    dn.max_rows = rows;
+    dn.group_rows_bound = rows;
+    return run_gemm(d, dn, EPI_PARTIAL, s);
+  }
   dn.max_rows = rows;
   dn.group_rows_bound = routed ? rows : d->T;
   dn.g_active = routed ? g_active : 0;
@@ -603,7 +646,11 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   void* zbuf = (desc->r > 0) ? (Z ? Z : ws + L.z) : nullptr;
   uint8_t* xa = ws + L.xa;  // [n + T, d]: expert-ordered rows, then X_hat
   void* h = ws + L.h;
-  const bool direct = (k == 1 && desc->n_shared == 0);
+  int n_allowed = 0;
+  for (int e = 0; e < desc->E; ++e) n_allowed += mask[e] ? 1 : 0;
+  const int split = splitk_factor(desc, n_allowed);
+  float* partial = split > 1 ? reinterpret_cast<float*>(ws + L.part) : nullptr;
+  const bool direct = (k == 1 && desc->n_shared == 0 && split == 1);
   void* slot = direct ? Y : static_cast<void*>(ws + L.slot);
   void* shared = desc->n_shared > 0 ? static_cast<void*>(ws + L.shared) : nullptr;
   int32_t* perm = reinterpret_cast<int32_t*>(ws + L.perm);
@@ -683,18 +730,21 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
     shared_a_rows = T;
     shared_a_base = 0;
   }
-  // Steps 4-5a: routed experts, gate scale and unpermute fused in the down projection.
-  int n_allowed = 0;
-  for (int e = 0; e < desc->E; ++e) n_allowed += mask[e] ? 1 : 0;
+  // Steps 4-5a: routed experts, gate scale and unpermute fused in the down
+  // projection (or in the split-K reduce).
   EC2MOE_CUDA(run_ffn(desc, true, xa, n + T, 0, offsets, w->W1, w->W3, w->W2, h, n + (long long)desc->n_shared * T, 0,
-                      perm, topk_w, slot, 0, stream, n_allowed));
+                      perm, topk_w, slot, 0, stream, n_allowed, partial, split));
   // Always-on shared experts on X_hat.
   if (desc->n_shared > 0) {
     EC2MOE_CUDA(run_ffn(desc, false, shared_a, shared_a_rows, shared_a_base, nullptr, w->W1s, w->W3s, w->W2s, h,
                         n + (long long)desc->n_shared * T, n, nullptr, nullptr, shared, 0, stream));
   }
   // Step 5b: fixed-order combine (skipped when the down projection wrote Y directly).
-  if (!direct) EC2MOE_CUDA(launch_combine(slot, shared, desc->n_shared, Y, desc->T, desc->k, desc->d, bf, stream));
+  if (split > 1)
+    EC2MOE_CUDA(launch_splitk_combine(partial, split, n, offsets, topk_idx, inv_perm, routed, topk_w, shared,
+                                      desc->n_shared, Y, desc->T, desc->k, desc->d, stream));
+  else if (!direct)
+    EC2MOE_CUDA(launch_combine(slot, shared, desc->n_shared, Y, desc->T, desc->k, desc->d, bf, stream));
   return EC2MOE_OK;
 }
 
@@ -768,7 +818,11 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
                              : nullptr;
     uint8_t* xa = ws + L.xa;
     void* h = ws + L.h;
-    const bool direct = (k == 1 && sub.n_shared == 0);
+    // the regions are sized for full micro-batches: split-K only where that
+    // layout holds the partial sums
+    const int split = splitk_possible(&full_sub) ? splitk_factor(&sub, n_allowed) : 1;
+    float* partial = split > 1 ? reinterpret_cast<float*>(ws + L.part) : nullptr;
+    const bool direct = (k == 1 && sub.n_shared == 0 && split == 1);
     void* slot = direct ? Yi : static_cast<void*>(ws + L.slot);
     void* shared = sub.n_shared > 0 ? static_cast<void*>(ws + L.shared) : nullptr;
     int32_t* perm = reinterpret_cast<int32_t*>(ws + L.perm);
@@ -826,11 +880,15 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
       shared_a_base = 0;
     }
     EC2MOE_CUDA(run_ffn(&sub, true, xa, n + T, 0, offsets, w->W1, w->W3, w->W2, h, n + (long long)sub.n_shared * T, 0,
-                        perm, tw_i, slot, 0, sc, n_allowed));
+                        perm, tw_i, slot, 0, sc, n_allowed, partial, split));
     if (sub.n_shared > 0)
       EC2MOE_CUDA(run_ffn(&sub, false, shared_a, shared_a_rows, shared_a_base, nullptr, w->W1s, w->W3s, w->W2s, h,
                           n + (long long)sub.n_shared * T, n, nullptr, nullptr, shared, 0, sc));
-    if (!direct) EC2MOE_CUDA(launch_combine(slot, shared, sub.n_shared, Yi, sub.T, sub.k, sub.d, bf, sc));
+    if (split > 1)
+      EC2MOE_CUDA(launch_splitk_combine(partial, split, n, offsets, idx_i, inv_perm, routed, tw_i, shared,
+                                        sub.n_shared, Yi, sub.T, sub.k, sub.d, sc));
+    else if (!direct)
+      EC2MOE_CUDA(launch_combine(slot, shared, sub.n_shared, Yi, sub.T, sub.k, sub.d, bf, sc));
   }
   // the layer's histogram is the sum of the micro-batches' ones
   EC2MOE_CUDA(launch_sum_counts(parts, used, desc->E, counts, sc));

@@ -112,12 +112,18 @@ cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long 
                           bool bf16, cudaStream_t s);
 // counts[e] = sum_p parts[p*E + e], p ascending.
 cudaError_t launch_sum_counts(const int32_t* parts, int n_parts, int E, int32_t* counts, cudaStream_t s);
+// Split-K expert output: y[t] = sum_slot w[t*k+slot] * sum_s partial[s][pos(t, slot)]
+// + sum_j shared[j*T+t], with pos = offsets[idx[i]] + rel[i] (rel_mode) or rel[i].
+cudaError_t launch_splitk_combine(const float* partial, int split_k, long long part_rows, const int32_t* offsets,
+                                  const int32_t* idx, const int32_t* rel, bool rel_mode, const float* w,
+                                  const void* shared, int n_shared, void* Y, int T, int k, int d, cudaStream_t s);
 // y[t] = sum_s slot[t*k+s] + sum_j shared[j*T+t]
 cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d,
                            bool bf16, cudaStream_t s);
 
 // ------------------------------------------------------------------ grouped GEMMs
-enum Epi { EPI_STORE = 0, EPI_GELU = 1, EPI_SWIGLU = 2, EPI_SCATTER = 3, EPI_REPLICATE = 4 };
+// EPI_PARTIAL: split-K partial sums, fp32, to partial[(split * part_rows + out_row) * N + col].
+enum Epi { EPI_STORE = 0, EPI_GELU = 1, EPI_SWIGLU = 2, EPI_SCATTER = 3, EPI_REPLICATE = 4, EPI_PARTIAL = 5 };
 
 // Group g of a grouped GEMM owns rows [row0(g), row0(g) + M_g) of A and of the
 // pre-scatter output, with
@@ -150,6 +156,9 @@ struct GemmArgs {
   long long max_rows;                // upper bound of sum_g M_g (for the grid size)
   int g_active;                      // groups expected to hold rows (tile-count estimate; 0 = G)
   long long group_rows_bound;        // upper bound of every M_g known on the host (0 = none)
+  int split_k;                       // EPI_PARTIAL: K ranges per output tile (1 = none)
+  float* partial;                    // EPI_PARTIAL: fp32 [split_k][part_rows][N]
+  long long part_rows;
   long long timeout_cycles;          // bounded-wait budget (tensor-core path)
   const char* name;                  // label for per-launch profiling (nullptr = by epilogue)
 };

@@ -373,6 +373,69 @@ cudaError_t launch_sum_counts(const int32_t* parts, int n_parts, int E, int32_t*
   return cudaGetLastError();
 }
 
+// Split-K expert outputs (bf16 layers): for every token and 8-column chunk,
+// the k slots' fp32 partial sums over the K ranges are added (range order),
+// weighted by the slot's gate weight (slot order), plus the shared experts'
+// rows; one bf16 rounding at the end.
+__global__ void splitk_combine_kernel(const float* __restrict__ partial, int S, long long part_rows,
+                                      const int32_t* __restrict__ offsets, const int32_t* __restrict__ idx,
+                                      const int32_t* __restrict__ rel, int rel_mode, const float* __restrict__ w,
+                                      const __nv_bfloat16* __restrict__ shared, int n_shared,
+                                      __nv_bfloat16* __restrict__ Y, int T, int k, int d) {
+  pdl_trigger();
+  pdl_wait();
+  const int per_row = d / 8;
+  const long long total = (long long)T * per_row;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (long long)gridDim.x * blockDim.x) {
+    const long long t = i / per_row;
+    const int c = static_cast<int>(i % per_row) * 8;
+    float acc[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[j] = 0.0f;
+    for (int slot = 0; slot < k; ++slot) {
+      const long long entry = t * k + slot;
+      const long long pos = rel_mode ? (long long)offsets[idx[entry]] + rel[entry] : (long long)rel[entry];
+      float sum[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) sum[j] = 0.0f;
+      for (int s = 0; s < S; ++s) {
+        float v[8];
+        load8(partial + ((long long)s * part_rows + pos) * d + c, v);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) sum[j] += v[j];
+      }
+      const float wt = w[entry];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] = fmaf(wt, sum[j], acc[j]);
+    }
+    for (int j = 0; j < n_shared; ++j) {
+      float v[8];
+      load8(shared + ((long long)j * T + t) * d + c, v);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) acc[q] += v[q];
+    }
+    store8(Y + t * d + c, acc);
+  }
+}
+
+cudaError_t launch_splitk_combine(const float* partial, int split_k, long long part_rows, const int32_t* offsets,
+                                  const int32_t* idx, const int32_t* rel, bool rel_mode, const float* w,
+                                  const void* shared, int n_shared, void* Y, int T, int k, int d, cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  const long long total = (long long)T * (d / 8);
+  long long blocks = (total + 255) / 256;
+  const long long cap = (long long)sm_count() * 8;
+  if (blocks > cap) blocks = cap;
+  KernelScope ks("combine", s);
+  cudaError_t e = launch_kernel(splitk_combine_kernel, dim3(static_cast<int>(blocks)), dim3(256), 0, s, partial, split_k,
+                                part_rows, offsets, idx, rel, rel_mode ? 1 : 0, w,
+                                static_cast<const __nv_bfloat16*>(shared), shared ? n_shared : 0,
+                                static_cast<__nv_bfloat16*>(Y), T, k, d);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
 cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d, bool bf16,
                            cudaStream_t s) {
   if (T <= 0) return cudaSuccess;

@@ -241,6 +241,7 @@ cudaError_t launch_r(const SkParams& p, int epi, int grid, cudaStream_t s) {
 // the tensor-core kernel's 128-row MMAs do almost no useful work and few
 // tiles exist; with more rows it streams the weights faster.
 bool gemm_skinny_supported(const GemmArgs& a, int epi) {
+  if (epi == EPI_PARTIAL) return false;
   const int limit = (epi == EPI_GELU || epi == EPI_SWIGLU) ? 2 : 4;
   return a.group_rows_bound > 0 && a.group_rows_bound <= limit && a.K % 8 == 0 && epi != EPI_REPLICATE &&
          (reinterpret_cast<uintptr_t>(a.A) % 16 == 0) && (reinterpret_cast<uintptr_t>(a.B) % 16 == 0) &&

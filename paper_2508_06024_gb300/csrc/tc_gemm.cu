@@ -68,6 +68,9 @@ struct Params {
   int rep_E;
   long long timeout;
   int n_tiles_n;
+  int split_k, kb_per_split;
+  float* partial;
+  long long part_rows;
 };
 
 // ------------------------------------------------------------------ tile schedule
@@ -193,7 +196,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   tc_fence_after();
   pdl_wait();
   const uint32_t tmem_base = *tmem_slot;
-  const int n_tiles = tile_prefix[p.G] * p.n_tiles_n;
+  // Split-K (EPI_PARTIAL): tile t covers output tile t / split_k and the
+  // k-blocks [ks * kb_per_split, ...) with ks = t % split_k.
+  const int n_tiles = tile_prefix[p.G] * p.n_tiles_n * p.split_k;
   const int num_kb = (p.K + BK - 1) / BK;
   const long long budget = p.timeout;
 
@@ -207,11 +212,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int cursor = 0;
       bool ok = true;
       for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        const TileCoord tc = decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
+        const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
         const int a_row = static_cast<int>(p.a_row_base) + (p.offsets ? row0[tc.g] : (p.a_shared ? 0 : row0[tc.g])) +
                           tc.m_blk * BM;
         const int b_row = tc.g * p.b_group_rows + tc.n_blk * C::BN_OUT;
-        for (int kb = 0; kb < num_kb; ++kb) {
+        const int kb0 = (tile % p.split_k) * p.kb_per_split;
+        const int kb1 = kb0 + p.kb_per_split < num_kb ? kb0 + p.kb_per_split : num_kb;
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1u, budget, abort_flag, &g_tc_error)) {
             ok = false;
             break;
@@ -255,7 +262,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int cursor = 0;
       bool ok = true, any = false;
       for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++it) {
-        (void)decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
+        (void)decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
+        const int kb0 = (tile % p.split_k) * p.kb_per_split;
+        const int kb1 = kb0 + p.kb_per_split < num_kb ? kb0 + p.kb_per_split : num_kb;
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
         if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, budget, abort_flag, &g_tc_error)) {
@@ -264,7 +273,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-        for (int kb = 0; kb < num_kb; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(full0 + 8u * stage, phase, budget, abort_flag, &g_tc_error)) {
             ok = false;
             break;
@@ -276,7 +285,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           // below 256 KB.
           const uint64_t da = da0 + static_cast<uint64_t>(stage) * DA_STAGE;
           const uint64_t db = db0 + static_cast<uint64_t>(stage) * DB_STAGE;
-          umma_bf16(d_tmem, da, db, IDESC, kb != 0 ? 1u : 0u);
+          umma_bf16(d_tmem, da, db, IDESC, kb != kb0 ? 1u : 0u);
 #pragma unroll
           for (int kk = 1; kk < BK / UK; ++kk) umma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, IDESC, 1u);
           any = true;
@@ -303,7 +312,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     int it = 0;
     int cursor = 0;
     for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++it) {
-      const TileCoord tc = decode_tile(tile, tile_prefix, p.n_tiles_n, cursor);
+      const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
+      const int ks = tile % p.split_k;
+      (void)ks;
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       // Row metadata first: its global loads overlap the tile's main loop.
@@ -377,6 +388,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int i = 0; i < C::CW; ++i) v[i] *= sc;
         }
         if (col >= p.N) continue;  // uniform across the warp
+        if (EPI == EPI_PARTIAL) {
+          // fp32 partial sums, 64 contiguous bytes per row and chunk
+          if (valid) {
+            float4* dstp = reinterpret_cast<float4*>(p.partial + (ks * p.part_rows + out_row) * p.N + col);
+#pragma unroll
+            for (int j = 0; j < C::CW / 4; ++j) dstp[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+          }
+          continue;
+        }
         __syncwarp();
 #pragma unroll
         for (int j = 0; j < SEGS; ++j) {
@@ -552,8 +572,16 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   p.rep_E = a.rep_E;
   p.timeout = a.timeout_cycles;
   p.n_tiles_n = (a.N + C::BN_OUT - 1) / C::BN_OUT;
+  p.split_k = EPI == EPI_PARTIAL && a.split_k > 1 ? a.split_k : 1;
+  {
+    const int num_kb = (a.K + BK - 1) / BK;
+    p.kb_per_split = (num_kb + p.split_k - 1) / p.split_k;
+    p.split_k = (num_kb + p.kb_per_split - 1) / p.kb_per_split;  // no empty K range
+  }
+  p.partial = a.partial;
+  p.part_rows = a.part_rows;
   const long long m_tiles_max = a.max_rows / BM + a.G;
-  long long tiles = m_tiles_max * p.n_tiles_n;
+  long long tiles = m_tiles_max * p.n_tiles_n * p.split_k;
   int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
   if (grid < 1) grid = 1;
   KernelScope ks(a.name ? a.name : kernel_name(EPI), s);
@@ -630,6 +658,10 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
     case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, s);
     case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, s);
     case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, s);
+    case EPI_PARTIAL:
+      if (!a.partial || a.N % 4 != 0) return cudaErrorInvalidValue;
+      return bn >= 256 ? launch_cfg<256, EPI_PARTIAL, stages_for(256)>(a, s)
+                       : launch_cfg<128, EPI_PARTIAL, stages_for(128)>(a, s);
   }
   return cudaErrorInvalidValue;
 }
