@@ -386,6 +386,49 @@ cudaError_t run_codec(const ec2moe_layer_desc* d, bool encode, const void* in, c
   return run_gemm(d, g, EPI_STORE, s);
 }
 
+// Steps 4-5 of a layer call on one stream, after the expert-ordered rows
+// (xa), perm and offsets exist: routed experts (gate scale and unpermute in
+// the down projection, or split-K partial sums), the always-on shared
+// experts, and the fixed-order combine or the split-K reduce into Y.
+struct ExpertStage {
+  const void* xa;               // [n + T, d]: expert-ordered rows, then X_hat
+  const void* shared_a;         // rows the shared experts read
+  long long shared_a_rows, shared_a_base;
+  void* h;                      // hidden rows
+  void* slot;                   // per-slot outputs (== Y when direct)
+  void* shared;                 // shared experts' outputs
+  float* partial;               // split-K partial sums (split > 1)
+  int split;
+  bool direct, routed;
+  const int32_t* offsets;
+  const int32_t* perm;
+  const int32_t* inv_perm;
+  const int32_t* topk_idx;
+  const float* topk_w;
+  void* Y;
+  int n_allowed;
+};
+
+cudaError_t run_expert_stage(const ec2moe_layer_desc* d, const ec2moe_layer_weights* w, const ExpertStage& x,
+                             cudaStream_t s) {
+  const long long T = d->T, n = T * d->k;
+  const bool bf = is_bf16(d);
+  cudaError_t e = run_ffn(d, true, x.xa, n + T, 0, x.offsets, w->W1, w->W3, w->W2, x.h,
+                          n + (long long)d->n_shared * T, 0, x.perm, x.topk_w, x.slot, 0, s, x.n_allowed, x.partial,
+                          x.split);
+  if (e != cudaSuccess) return e;
+  if (d->n_shared > 0) {
+    e = run_ffn(d, false, x.shared_a, x.shared_a_rows, x.shared_a_base, nullptr, w->W1s, w->W3s, w->W2s, x.h,
+                n + (long long)d->n_shared * T, n, nullptr, nullptr, x.shared, 0, s);
+    if (e != cudaSuccess) return e;
+  }
+  if (x.split > 1)
+    return launch_splitk_combine(x.partial, x.split, n, x.offsets, x.topk_idx, x.inv_perm, x.routed, x.topk_w,
+                                 x.shared, d->n_shared, x.Y, d->T, d->k, d->d, s);
+  if (!x.direct) return launch_combine(x.slot, x.shared, d->n_shared, x.Y, d->T, d->k, d->d, bf, s);
+  return cudaSuccess;
+}
+
 // Argument checks of a whole-layer call (everything but the workspace).
 ec2moe_status check_layer_call(const ec2moe_layer_desc* desc, const ec2moe_layer_weights* w, const void* X,
                                const uint8_t* mask, void* Y, int32_t* topk_idx, float* topk_w, int32_t* counts,
@@ -730,21 +773,10 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
     shared_a_rows = T;
     shared_a_base = 0;
   }
-  // Steps 4-5a: routed experts, gate scale and unpermute fused in the down
-  // projection (or in the split-K reduce).
-  EC2MOE_CUDA(run_ffn(desc, true, xa, n + T, 0, offsets, w->W1, w->W3, w->W2, h, n + (long long)desc->n_shared * T, 0,
-                      perm, topk_w, slot, 0, stream, n_allowed, partial, split));
-  // Always-on shared experts on X_hat.
-  if (desc->n_shared > 0) {
-    EC2MOE_CUDA(run_ffn(desc, false, shared_a, shared_a_rows, shared_a_base, nullptr, w->W1s, w->W3s, w->W2s, h,
-                        n + (long long)desc->n_shared * T, n, nullptr, nullptr, shared, 0, stream));
-  }
-  // Step 5b: fixed-order combine (skipped when the down projection wrote Y directly).
-  if (split > 1)
-    EC2MOE_CUDA(launch_splitk_combine(partial, split, n, offsets, topk_idx, inv_perm, routed, topk_w, shared,
-                                      desc->n_shared, Y, desc->T, desc->k, desc->d, stream));
-  else if (!direct)
-    EC2MOE_CUDA(launch_combine(slot, shared, desc->n_shared, Y, desc->T, desc->k, desc->d, bf, stream));
+  // Steps 4-5: routed and shared experts, combine (or the split-K reduce).
+  const ExpertStage xs{xa, shared_a, shared_a_rows, shared_a_base, h, slot, shared, partial, split, direct, routed,
+                       offsets, perm, inv_perm, topk_idx, topk_w, Y, n_allowed};
+  EC2MOE_CUDA(run_expert_stage(desc, w, xs, stream));
   return EC2MOE_OK;
 }
 
@@ -879,16 +911,9 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
       shared_a_rows = T;
       shared_a_base = 0;
     }
-    EC2MOE_CUDA(run_ffn(&sub, true, xa, n + T, 0, offsets, w->W1, w->W3, w->W2, h, n + (long long)sub.n_shared * T, 0,
-                        perm, tw_i, slot, 0, sc, n_allowed, partial, split));
-    if (sub.n_shared > 0)
-      EC2MOE_CUDA(run_ffn(&sub, false, shared_a, shared_a_rows, shared_a_base, nullptr, w->W1s, w->W3s, w->W2s, h,
-                          n + (long long)sub.n_shared * T, n, nullptr, nullptr, shared, 0, sc));
-    if (split > 1)
-      EC2MOE_CUDA(launch_splitk_combine(partial, split, n, offsets, idx_i, inv_perm, routed, tw_i, shared,
-                                        sub.n_shared, Yi, sub.T, sub.k, sub.d, sc));
-    else if (!direct)
-      EC2MOE_CUDA(launch_combine(slot, shared, sub.n_shared, Yi, sub.T, sub.k, sub.d, bf, sc));
+    const ExpertStage xs{xa, shared_a, shared_a_rows, shared_a_base, h, slot, shared, partial, split, direct, routed,
+                         offsets, perm, inv_perm, idx_i, tw_i, Yi, n_allowed};
+    EC2MOE_CUDA(run_expert_stage(&sub, w, xs, sc));
   }
   // the layer's histogram is the sum of the micro-batches' ones
   EC2MOE_CUDA(launch_sum_counts(parts, used, desc->E, counts, sc));
