@@ -723,7 +723,8 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
     if (gate_split_bytes(desc->E, desc->n_groups, desc->d, bf)) ga.w_split = ws + L.wsplit;
   }
   bool routed = false;
-  EC2MOE_CUDA(launch_gate(ga, bf, stream, &routed));
+  int gate_sms = 0;
+  EC2MOE_CUDA(launch_gate(ga, bf, stream, &routed, &gate_sms));
   // Step 3b: routing tables (inside the gate kernel when it could take them).
   if (!routed) EC2MOE_CUDA(launch_route(topk_idx, n, desc->E, blk, counts, offsets, perm, inv_perm, stream));
   RelPlace rel;
@@ -758,6 +759,7 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
     ca.offsets_out = offsets;
     ca.self_row_base = desc->n_shared > 0 ? n : -1;
     ca.timeout_cycles = default_timeout_cycles();
+    ca.busy_sms = gate_sms;
     EC2MOE_CUDA(launch_codec_fused(ca, stream));
   } else if (desc->r > 0) {
     EC2MOE_CUDA(run_codec(desc, true, X, w->V_enc, zbuf, stream));

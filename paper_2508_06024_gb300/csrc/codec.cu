@@ -394,19 +394,27 @@ cudaError_t launch_bn_r(const CodecArgs& a, cudaStream_t s) {
 
 template <int R>
 cudaError_t launch_r(const CodecArgs& a, cudaStream_t s) {
-  // d-chunk width: the widest whose CTA count fills the most of the GPU in one wave
+  // d-chunk width: the widest whose CTA count fills the most of the GPU in one
+  // wave.  The kernel runs under programmatic dependent launch next to the
+  // gate kernel, whose CTAs hold `busy_sms` SMs until it ends; a grid that
+  // fits in the other SMs runs both GEMMs while the gate runs, while CTAs
+  // beyond them would start only after it, on the critical path.
   const int m_tiles = (a.T + BM - 1) / BM;
   const int sms = sm_count();
+  const int free_sms = sms - (a.busy_sms > 0 && a.busy_sms < sms ? a.busy_sms : 0);
   const int cands[3] = {256, 192, 128};
   int best = 256;
   double best_eff = -1.0;
-  for (int bn : cands) {
-    const long long ctas = (long long)m_tiles * ((a.d + bn - 1) / bn);
-    const long long waves = (ctas + sms - 1) / sms;
-    const double eff = (double)ctas / (double)(waves * sms) * (bn == 256 ? 1.0 : (bn == 192 ? 0.98 : 0.95));
-    if (eff > best_eff + 1e-9) {
-      best_eff = eff;
-      best = bn;
+  for (int pass = 0; pass < 2 && best_eff < 0.0; ++pass) {
+    for (int bn : cands) {
+      const long long ctas = (long long)m_tiles * ((a.d + bn - 1) / bn);
+      if (pass == 0 && ctas > free_sms) continue;  // first choice: fits beside the gate
+      const long long waves = (ctas + sms - 1) / sms;
+      const double eff = (double)ctas / (double)(waves * sms) * (bn == 256 ? 1.0 : (bn == 192 ? 0.98 : 0.95));
+      if (eff > best_eff + 1e-9) {
+        best_eff = eff;
+        best = bn;
+      }
     }
   }
   switch (best) {

@@ -671,8 +671,11 @@ __global__ void __launch_bounds__(SL_THREADS) gate_tiled_kernel(const KParams p)
 
 }  // namespace
 
-cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed) {
+cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed, int* held_sms) {
   if (routed) *routed = false;
+  // The SIMT gates launch at least one CTA per SM once the batch fills the
+  // GPU; counted as holding every SM.
+  if (held_sms) *held_sms = sm_count();
   KParams p;
   p.X = a.X;
   p.W_local = a.W_local;
@@ -694,7 +697,7 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* rout
   cudaError_t e;
   {
     bool handled = false;
-    e = launch_gate_tensor(a, p, O, bf16, s, routed, &handled);
+    e = launch_gate_tensor(a, p, O, bf16, s, routed, held_sms, &handled);
     if (handled || e != cudaSuccess) return e;
   }
   // Slice kernel when every gate row fits in shared memory next to the

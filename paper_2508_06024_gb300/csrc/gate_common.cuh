@@ -29,7 +29,7 @@ struct KParams {
 
 // Tensor-core gate (bf16, at most 80 gate rows) with its prep kernel; sets
 // *handled when it took the call (else the caller runs a SIMT gate).
-cudaError_t launch_gate_tensor(const GateArgs& a, KParams p, int O, bool bf16, cudaStream_t s, bool* routed,
+cudaError_t launch_gate_tensor(const GateArgs& a, KParams p, int O, bool bf16, cudaStream_t s, bool* routed, int* held_sms,
                                bool* handled);
 
 }  // namespace gatek

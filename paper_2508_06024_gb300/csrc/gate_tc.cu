@@ -745,7 +745,7 @@ cudaError_t launch_gate_tc(const KParams& p, int stages, cudaStream_t s, const C
 
 }  // namespace
 
-cudaError_t launch_gate_tensor(const GateArgs& a, KParams p, int O, bool bf16, cudaStream_t s, bool* routed,
+cudaError_t launch_gate_tensor(const GateArgs& a, KParams p, int O, bool bf16, cudaStream_t s, bool* routed, int* held_sms,
                                bool* handled) {
   *handled = false;
   cudaError_t e = cudaSuccess;
@@ -794,6 +794,10 @@ cudaError_t launch_gate_tensor(const GateArgs& a, KParams p, int O, bool bf16, c
         if (e != cudaSuccess) return e;
       }
       KernelScope ks("gate_topk", s);
+      if (held_sms) {  // one CTA per SM (the kernel's shared memory allows no second)
+        const int n_tiles = (a.T + GC_BM - 1) / GC_BM;
+        *held_sms = n_tiles < sm_count() ? n_tiles : sm_count();
+      }
       e = prep ? launch_gate_tc<true>(p, stages, s, mX, mW, mWg) : launch_gate_tc<false>(p, stages, s, mX, mW, mWg);
       if (e != cudaSuccess) return e;
       return cudaGetLastError();

@@ -87,8 +87,10 @@ struct GateArgs {
 // Bytes of the prepared split gate rows (0 when the tensor-core gate does not apply).
 size_t gate_split_bytes(int E, int K, int d, bool bf16);
 // Launches the gate; with the routing fields set, also fills them when the
-// fused path applies (*routed = true), else gate only.
-cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed = nullptr);
+// fused path applies (*routed = true), else gate only.  *held_sms (optional)
+// receives how many SMs the gate kernel's CTAs occupy while it runs.
+cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed = nullptr,
+                        int* held_sms = nullptr);
 // Rows into expert order from relative positions: for entry i (token i / k),
 // pos = offsets[e] + rel[i] with offsets = exclusive prefix of counts;
 // dst[pos] = src[i / k], perm[pos] = i; block 0 writes offsets[0..E].
@@ -192,6 +194,7 @@ struct CodecArgs {
   int32_t* offsets_out;    // [E+1]
   long long self_row_base;
   long long timeout_cycles;
+  int busy_sms;            // SMs held by the kernel this one overlaps (the gate): the grid is sized to the rest
 };
 bool codec_fused_supported(int d, int r);
 cudaError_t launch_codec_fused(const CodecArgs& a, cudaStream_t s);
