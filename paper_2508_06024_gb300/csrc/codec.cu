@@ -281,16 +281,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     // Routing metadata comes from the gate kernel: wait for it here only.
     pdl_wait();
-    if (warp == 2 && lane == 0) {
-      int run = 0;
-      for (int e = 0; e < p.E; ++e) {
-        s_off[e] = run;
-        run += p.counts[e];
-      }
-      s_off[p.E] = run;
-      if (blockIdx.x == 0)
-        for (int e = 0; e <= p.E; ++e) p.offsets_out[e] = s_off[e];
-    }
+    if (warp == 2)
+      warp_exclusive_scan<5>(p.E, lane, [&](int e) { return p.counts[e]; }, s_off,
+                             blockIdx.x == 0 ? p.offsets_out : nullptr);
     asm volatile("bar.sync 1, %0;" ::"r"(EPI_WARPS * 32) : "memory");
     int rdst[8];
 #pragma unroll
@@ -310,43 +303,47 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       constexpr int SEGS = C::CW / 8;
       constexpr int ROWS_PER_PASS = 32 / SEGS;
       constexpr int NCH = C::PART_X / C::CW;
+      // Two 16-column chunks per TMEM round trip; the slot loop is unrolled so
+      // both register buffers stay in registers (a runtime index into them
+      // would place them in local memory).
       uint32_t rv[2][C::CW];
 #pragma unroll 1
-      for (int ci = 0; ci < NCH; ++ci) {
-        const int c0 = part * C::PART_X + ci * C::CW;
-        const int slot = ci & 1;
-        if (slot == 0) {
-          tmem_ld16_nw(t_row + X_ACC_COL + c0, rv[0]);
-          if (ci + 1 < NCH) tmem_ld16_nw(t_row + X_ACC_COL + c0 + C::CW, rv[1]);
-          tmem_wait();
-        }
-        const int col = n0 + c0;
-        if (col >= p.d) continue;  // uniform across the warp
-        __syncwarp();
+      for (int cp = 0; cp < NCH; cp += 2) {
+        tmem_ld16_nw(t_row + X_ACC_COL + part * C::PART_X + cp * C::CW, rv[0]);
+        if (cp + 1 < NCH) tmem_ld16_nw(t_row + X_ACC_COL + part * C::PART_X + (cp + 1) * C::CW, rv[1]);
+        tmem_wait();
 #pragma unroll
-        for (int j = 0; j < SEGS; ++j) {
-          const uint32_t* rr = slot ? rv[1] : rv[0];
-          U4 q4{pack_bf16x2(__uint_as_float(rr[8 * j + 0]), __uint_as_float(rr[8 * j + 1])),
-                pack_bf16x2(__uint_as_float(rr[8 * j + 2]), __uint_as_float(rr[8 * j + 3])),
-                pack_bf16x2(__uint_as_float(rr[8 * j + 4]), __uint_as_float(rr[8 * j + 5])),
-                pack_bf16x2(__uint_as_float(rr[8 * j + 6]), __uint_as_float(rr[8 * j + 7]))};
-          *reinterpret_cast<U4*>(stg + lane * C::STG_PITCH + 16 * j) = q4;
-        }
-        __syncwarp();
-        const int sg = lane % SEGS;
+        for (int slot = 0; slot < 2; ++slot) {
+          if (cp + slot >= NCH) break;
+          const int c0 = part * C::PART_X + (cp + slot) * C::CW;
+          const int col = n0 + c0;
+          if (col >= p.d) break;  // uniform across the warp; later chunks lie further right
+          __syncwarp();
 #pragma unroll
-        for (int pass = 0; pass < SEGS; ++pass) {
-          const int rr_row = pass * ROWS_PER_PASS + lane / SEGS;
-          const bool rvalid = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr_row) != 0;
-          const long long grow_r = __shfl_sync(0xffffffffu, grow, rr_row);
-          const U4 q4 = *reinterpret_cast<const U4*>(stg + rr_row * C::STG_PITCH + 16 * sg);
-#pragma unroll
-          for (int r = 0; r < 8; ++r) {
-            const int dr = __shfl_sync(0xffffffffu, rdst[r], rr_row);
-            if (rvalid && r < p.k) *reinterpret_cast<U4*>(p.out + (long long)dr * p.ldo + col + 8 * sg) = q4;
+          for (int j = 0; j < SEGS; ++j) {
+            const uint32_t* rr = rv[slot];
+            U4 q4{pack_bf16x2(__uint_as_float(rr[8 * j + 0]), __uint_as_float(rr[8 * j + 1])),
+                  pack_bf16x2(__uint_as_float(rr[8 * j + 2]), __uint_as_float(rr[8 * j + 3])),
+                  pack_bf16x2(__uint_as_float(rr[8 * j + 4]), __uint_as_float(rr[8 * j + 5])),
+                  pack_bf16x2(__uint_as_float(rr[8 * j + 6]), __uint_as_float(rr[8 * j + 7]))};
+            *reinterpret_cast<U4*>(stg + lane * C::STG_PITCH + 16 * j) = q4;
           }
-          if (rvalid && p.self_row_base >= 0)
-            *reinterpret_cast<U4*>(p.out + (p.self_row_base + grow_r) * p.ldo + col + 8 * sg) = q4;
+          __syncwarp();
+          const int sg = lane % SEGS;
+#pragma unroll
+          for (int pass = 0; pass < SEGS; ++pass) {
+            const int rr_row = pass * ROWS_PER_PASS + lane / SEGS;
+            const bool rvalid = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr_row) != 0;
+            const long long grow_r = __shfl_sync(0xffffffffu, grow, rr_row);
+            const U4 q4 = *reinterpret_cast<const U4*>(stg + rr_row * C::STG_PITCH + 16 * sg);
+#pragma unroll
+            for (int r = 0; r < 8; ++r) {
+              const int dr = __shfl_sync(0xffffffffu, rdst[r], rr_row);
+              if (rvalid && r < p.k) *reinterpret_cast<U4*>(p.out + (long long)dr * p.ldo + col + 8 * sg) = q4;
+            }
+            if (rvalid && p.self_row_base >= 0)
+              *reinterpret_cast<U4*>(p.out + (p.self_row_base + grow_r) * p.ldo + col + 8 * sg) = q4;
+          }
         }
       }
     }

@@ -71,4 +71,38 @@ __device__ __forceinline__ float gelu_bf16out(float u) {
 // SiLU for bf16-output epilogues: fast exp and division (relative error ~1e-7).
 __device__ __forceinline__ float silu_bf16out(float u) { return __fdividef(u, 1.0f + __expf(-u)); }
 
+// Exclusive prefix sum of n <= 32 * CHUNKS values by one warp (all 32 lanes
+// call it): out[i] = value(0) + ... + value(i - 1) for i <= n, so out[n] is
+// the total, which every lane returns.  All values are fetched before the
+// scan, so reading them from global memory costs about one memory latency
+// instead of n dependent ones.  copy (optional, global) receives out[0..n].
+template <int CHUNKS, typename F>
+__device__ __forceinline__ int warp_exclusive_scan(int n, int lane, F value, int* out, int* copy = nullptr) {
+  int v[CHUNKS];
+#pragma unroll
+  for (int c = 0; c < CHUNKS; ++c) v[c] = c * 32 + lane < n ? value(c * 32 + lane) : 0;
+  int carry = 0;
+#pragma unroll
+  for (int c = 0; c < CHUNKS; ++c) {
+    if (c * 32 >= n) break;  // uniform
+    int x = v[c];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, x, o);
+      if (lane >= o) x += y;
+    }
+    const int i = c * 32 + lane;
+    if (i < n) {
+      out[i] = carry + x - v[c];
+      if (copy) copy[i] = carry + x - v[c];
+    }
+    carry += __shfl_sync(0xffffffffu, x, 31);
+  }
+  if (lane == 0) {
+    out[n] = carry;
+    if (copy) copy[n] = carry;
+  }
+  return carry;
+}
+
 }  // namespace ec2moe

@@ -211,18 +211,11 @@ __global__ void gather_rel_kernel(const uint8_t* __restrict__ src, uint8_t* __re
   pdl_trigger();
   pdl_wait();
   __shared__ int s_off[MAXE + 1];
-  if (threadIdx.x == 0) {
-    int run = 0;
-    for (int e = 0; e < E; ++e) {
-      s_off[e] = run;
-      run += counts[e];
-    }
-    s_off[E] = run;
-    if (blockIdx.x == 0)
-      for (int e = 0; e <= E; ++e) offsets[e] = s_off[e];
-  }
-  __syncthreads();
   const int lane = threadIdx.x & 31;
+  if (threadIdx.x < 32)
+    warp_exclusive_scan<(MAXE + 31) / 32>(E, lane, [&](int e) { return counts[e]; }, s_off,
+                                          blockIdx.x == 0 ? offsets : nullptr);
+  __syncthreads();
   const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
   for (long long i = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < n; i += warps) {
     const int pos = s_off[idx[i]] + rel[i];

@@ -152,33 +152,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 0) {
     pdl_wait();
-    // Per-group tile prefix (m tiles) and first rows.
-    int acc = 0;
-    tile_prefix[0] = 0;
-    for (int g = 0; g < p.G; ++g) {
-      int r0, mg;
-      if (p.offsets) {
-        r0 = p.offsets[g];
-        mg = p.offsets[g + 1] - r0;
-      } else {
-        r0 = g * p.M;
-        mg = p.M;
-      }
-      row0[g] = r0;
-      acc += (mg + BM - 1) / BM;
-      tile_prefix[g + 1] = acc;
-    }
-    if (EPI == EPI_REPLICATE && p.rep_counts) {
-      int run = 0;
-      for (int e = 0; e < p.rep_E; ++e) {
-        s_off[e] = run;
-        run += p.rep_counts[e];
-      }
-      s_off[p.rep_E] = run;
-      if (blockIdx.x == 0)
-        for (int e = 0; e <= p.rep_E; ++e) p.rep_offsets_out[e] = s_off[e];
-    }
+    // Per-group first rows and tile prefix (m tiles), one warp-wide scan.
+    warp_exclusive_scan<(MAX_GROUPS + 31) / 32>(
+        p.G, lane,
+        [&](int g) {
+          int r0 = g * p.M, mg = p.M;
+          if (p.offsets) {
+            r0 = p.offsets[g];
+            mg = p.offsets[g + 1] - r0;
+          }
+          row0[g] = r0;
+          return (mg + BM - 1) / BM;
+        },
+        tile_prefix);
+    if (EPI == EPI_REPLICATE && p.rep_counts)
+      warp_exclusive_scan<(MAX_GROUPS + 31) / 32>(p.rep_E, lane, [&](int e) { return p.rep_counts[e]; }, s_off,
+                                                   blockIdx.x == 0 ? p.rep_offsets_out : nullptr);
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tmA);
