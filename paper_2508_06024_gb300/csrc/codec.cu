@@ -8,10 +8,12 @@
 //      to global (chunk 0's CTA) and into shared memory in the swizzled
 //      K-major layout the second MMA reads as its A operand;
 //   3. X_hat chunk = Z_tile V_dec[chunk]^T (N = BN) into TMEM;
-//   4. each X_hat row goes straight to its (token, slot) positions in expert
-//      order (offsets[e] + the row's position relative to its expert, from
-//      the routing the gate kernel filled), and to the tail rows the shared
-//      experts read.
+//   4. the X_hat chunk is rounded to bf16 into a row-major tile in the
+//      (then idle) pipeline buffers, and each epilogue warp copies whole row
+//      segments (BN * 2 contiguous bytes) to the row's (token, slot)
+//      positions in expert order (offsets[e] + the row's position relative
+//      to its expert, from the routing the gate kernel filled) and to the
+//      tail rows the shared experts read.
 // Z is recomputed by the d / BN CTAs of a token tile (cheap at r <= 256);
 // nothing but the routing metadata depends on the previous kernel, so under
 // programmatic dependent launch both GEMMs run before griddepcontrol.wait.
@@ -69,16 +71,18 @@ struct CCfg {
   static constexpr int PART_X = BN / PARTS_X;                  // X_hat columns per epilogue warp
   static constexpr int PART_Z = R / 4;                         // Z columns per epilogue warp
   static constexpr int CW = 16;
-  static constexpr int STG_PITCH = CW * 2 + 16;
-  static constexpr int STG_BYTES = EPI_WARPS * 32 * STG_PITCH;
+  static constexpr int TILE_PITCH = BN * 2 + 16;               // bf16 X_hat tile row (padded against bank conflicts)
+  static constexpr int DST_BYTES = BM * 8 * 4;                 // destination rows of each tile row (k <= 8)
   static constexpr int MISC = 1024;                            // barriers, TMEM slot, flags, offsets
-  static constexpr int FIXED = 1024 + Z_BYTES + STG_BYTES + MISC;
+  static constexpr int FIXED = 1024 + Z_BYTES + DST_BYTES + MISC;
   static constexpr int STAGES_FIT = (220 * 1024 - FIXED) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 4 ? 4 : STAGES_FIT;
   static constexpr int SMEM = FIXED + STAGES * STAGE_BYTES;
   static_assert(STAGES >= 2, "codec pipeline needs two stages");
   static_assert(SMEM <= 232448, "shared memory per CTA");
   static_assert(PART_X % CW == 0 && PART_Z % CW == 0 && R % 64 == 0, "column split");
+  static_assert(STAGES * STAGE_BYTES >= BM * TILE_PITCH, "X_hat tile fits in the pipeline buffers");
+  static_assert(BN <= 256, "one 16-byte piece per lane covers a row segment");
 };
 
 template <int BN, int R>
@@ -90,8 +94,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* stages = smem;
   uint8_t* zs = smem + C::STAGES * C::STAGE_BYTES;
-  uint8_t* stg_all = zs + C::Z_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(stg_all + C::STG_BYTES);
+  int* s_dst = reinterpret_cast<int*>(zs + C::Z_BYTES);  // [BM][8]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(zs + C::Z_BYTES + C::DST_BYTES);
   uint64_t* full = bars;
   uint64_t* empty = bars + C::STAGES;
   uint64_t* zfull = bars + 2 * C::STAGES;
@@ -285,27 +289,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       warp_exclusive_scan<5>(p.E, lane, [&](int e) { return p.counts[e]; }, s_off,
                              blockIdx.x == 0 ? p.offsets_out : nullptr);
     asm volatile("bar.sync 1, %0;" ::"r"(EPI_WARPS * 32) : "memory");
-    int rdst[8];
+    // Destination rows of this tile row (one thread per row writes them).
+    if (part == 0) {
 #pragma unroll
-    for (int r = 0; r < 8; ++r) {
-      rdst[r] = 0;
-      if (valid && r < p.k) {
-        const long long entry = grow * p.k + r;
-        const int dst = s_off[p.topk_idx[entry]] + p.rel[entry];
-        if (n_chunk == 0) p.perm_out[dst] = static_cast<int32_t>(entry);
-        rdst[r] = dst;
+      for (int r = 0; r < 8; ++r) {
+        if (valid && r < p.k) {
+          const long long entry = grow * p.k + r;
+          const int dst = s_off[p.topk_idx[entry]] + p.rel[entry];
+          if (n_chunk == 0) p.perm_out[dst] = static_cast<int32_t>(entry);
+          s_dst[row * 8 + r] = dst;
+        }
       }
     }
     if (ok) ok = mbar_wait(smem_u32(xfull), 0, budget, abort_flag, &g_codec_error);
     if (ok) {
+      // Every MMA has completed, so the pipeline buffers are free: round this
+      // warp's 32 rows x PART_X columns into the row-major bf16 tile.
       tc_fence_after();
-      uint8_t* stg = stg_all + (warp - 2) * 32 * C::STG_PITCH;
-      constexpr int SEGS = C::CW / 8;
-      constexpr int ROWS_PER_PASS = 32 / SEGS;
       constexpr int NCH = C::PART_X / C::CW;
-      // Two 16-column chunks per TMEM round trip; the slot loop is unrolled so
-      // both register buffers stay in registers (a runtime index into them
-      // would place them in local memory).
+      uint8_t* trow = stages + row * C::TILE_PITCH + part * C::PART_X * 2;
       uint32_t rv[2][C::CW];
 #pragma unroll 1
       for (int cp = 0; cp < NCH; cp += 2) {
@@ -315,35 +317,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
         for (int slot = 0; slot < 2; ++slot) {
           if (cp + slot >= NCH) break;
-          const int c0 = part * C::PART_X + (cp + slot) * C::CW;
-          const int col = n0 + c0;
-          if (col >= p.d) break;  // uniform across the warp; later chunks lie further right
-          __syncwarp();
+          const uint32_t* rr = rv[slot];
 #pragma unroll
-          for (int j = 0; j < SEGS; ++j) {
-            const uint32_t* rr = rv[slot];
+          for (int j = 0; j < C::CW / 8; ++j) {
             U4 q4{pack_bf16x2(__uint_as_float(rr[8 * j + 0]), __uint_as_float(rr[8 * j + 1])),
                   pack_bf16x2(__uint_as_float(rr[8 * j + 2]), __uint_as_float(rr[8 * j + 3])),
                   pack_bf16x2(__uint_as_float(rr[8 * j + 4]), __uint_as_float(rr[8 * j + 5])),
                   pack_bf16x2(__uint_as_float(rr[8 * j + 6]), __uint_as_float(rr[8 * j + 7]))};
-            *reinterpret_cast<U4*>(stg + lane * C::STG_PITCH + 16 * j) = q4;
+            *reinterpret_cast<U4*>(trow + ((cp + slot) * C::CW + 8 * j) * 2) = q4;
           }
-          __syncwarp();
-          const int sg = lane % SEGS;
-#pragma unroll
-          for (int pass = 0; pass < SEGS; ++pass) {
-            const int rr_row = pass * ROWS_PER_PASS + lane / SEGS;
-            const bool rvalid = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr_row) != 0;
-            const long long grow_r = __shfl_sync(0xffffffffu, grow, rr_row);
-            const U4 q4 = *reinterpret_cast<const U4*>(stg + rr_row * C::STG_PITCH + 16 * sg);
-#pragma unroll
-            for (int r = 0; r < 8; ++r) {
-              const int dr = __shfl_sync(0xffffffffu, rdst[r], rr_row);
-              if (rvalid && r < p.k) *reinterpret_cast<U4*>(p.out + (long long)dr * p.ldo + col + 8 * sg) = q4;
-            }
-            if (rvalid && p.self_row_base >= 0)
-              *reinterpret_cast<U4*>(p.out + (p.self_row_base + grow_r) * p.ldo + col + 8 * sg) = q4;
-          }
+        }
+      }
+      tc_fence_before();
+    }
+    // The tile is complete unless a wait of some warp timed out, which set
+    // the abort flag before this barrier.
+    asm volatile("bar.sync 1, %0;" ::"r"(EPI_WARPS * 32) : "memory");
+    if (ok && !*abort_flag) {
+      // Row segments: warp w copies rows w, w + 16, ...; lane l carries
+      // columns n0 + 8l .. +7 (16 bytes), so a row segment is one coalesced
+      // store per destination.
+      const int ew = warp - 2;
+      const int col = n0 + 8 * lane;
+      const bool lane_on = 8 * lane < BN && col < p.d;
+#pragma unroll 1
+      for (int tr = ew; tr < BM; tr += EPI_WARPS) {
+        const long long g = m0 + tr;
+        if (g >= p.T) break;  // uniform; later rows are further out
+        if (lane_on) {
+          const U4 q4 = *reinterpret_cast<const U4*>(stages + tr * C::TILE_PITCH + 16 * lane);
+          for (int r = 0; r < p.k; ++r)
+            *reinterpret_cast<U4*>(p.out + (long long)s_dst[tr * 8 + r] * p.ldo + col) = q4;
+          if (p.self_row_base >= 0) *reinterpret_cast<U4*>(p.out + (p.self_row_base + g) * p.ldo + col) = q4;
         }
       }
     }
