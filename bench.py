@@ -116,6 +116,13 @@ def kernel_work(cfg, name: str, touched: int = 0):
         return 2.0 * T * r * d, es * (T * r + d * r + rows_out * d)
     if name == "lr_codec":
         return 4.0 * T * d * r, es * (T * d + 2 * r * d + T * r + n * d)
+    if name == "gate_decide":
+        # the small-batch gate's second kernel: partial logits in (not layer
+        # work), Top-k ids and weights out
+        return 0.0, 8 * n
+    if name == "lr_reduce":
+        # the split-K encoder's reduce: its fp32 partial sums are not layer work
+        return 0.0, es * T * r
     if name == "gate_topk":
         return 2.0 * T * d * (E + K), es * T * d + 4 * (E + K) * d + 8 * n
     if name == "gate_prep":
@@ -543,7 +550,8 @@ def run_ours(args):
     return 0
 
 
-END_STAGE = ("gate_prep", "gate_topk", "lr_encode", "route", "route_count", "route_scatter")
+END_STAGE = ("gate_prep", "gate_topk", "gate_decide", "lr_encode", "lr_reduce", "route", "route_count",
+             "route_scatter")
 
 
 def run_pipeline(args):

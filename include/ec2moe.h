@@ -288,9 +288,9 @@ int32_t ec2moe_last_launch_count(void);
  * bracketed by a pair of CUDA events recorded on its stream; records
  * accumulate until ec2moe_profile_reset.  Reading a record synchronises on its
  * stop event.  `name` receives a static string naming the launch
- * ("gate_prep", "gate_topk", "route_count", "route_scatter", "gather_rows", "lr_encode",
- * "lr_decode", "expert_up", "expert_down", "shared_up", "shared_down",
- * "combine", "sum_counts"); `ms` its device duration.  Profiling is off by default and
+ * ("gate_prep", "gate_topk", "gate_decide", "route_count", "route_scatter", "gather_rows",
+ * "lr_encode", "lr_reduce", "lr_decode", "lr_codec", "expert_up", "expert_down", "shared_up",
+ * "shared_down", "combine", "sum_counts"); `ms` its device duration.  Profiling is off by default and
  * costs nothing when off. */
 ec2moe_status ec2moe_profile_enable(int32_t enable);
 int32_t ec2moe_profile_count(void);

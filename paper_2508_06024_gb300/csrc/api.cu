@@ -231,8 +231,26 @@ int splitk_factor(const ec2moe_layer_desc* d, int n_allowed) {
   return best;
 }
 
+// Split-K encoder for decode-sized batches: with T <= 256 rows the encoder
+// has at most 2 x (r / 128) output tiles over K = d_model, so one CTA per tile
+// would stream V_enc alone; the K range is split (at least two k-blocks of 64
+// per range, at most 32 ranges, about one unit per SM) and one small kernel
+// adds the fp32 partial sums into Z.
+constexpr int ENC_SPLIT_MAX = 32;
+int enc_split(const ec2moe_layer_desc* d) {
+  if (!is_bf16(d) || d->r <= 0 || d->r % 128 != 0 || d->T > 256 || d->d < 1024) return 1;
+  const long long tiles = (long long)((d->T + 127) / 128) * (d->r / 128);
+  long long s = sm_count() / tiles;
+  if (s > d->d / 128) s = d->d / 128;
+  if (s > ENC_SPLIT_MAX) s = ENC_SPLIT_MAX;
+  if (s < 2) return 1;
+  // the count of non-empty ranges the GEMM derives from this request
+  const long long nk = (d->d + 63) / 64, per = (nk + s - 1) / s;
+  return static_cast<int>((nk + per - 1) / per);
+}
+
 struct LayerWs {
-  size_t z, xa, h, slot, shared, perm, inv_perm, offsets, blk, wsplit, part, total;
+  size_t z, xa, h, slot, shared, perm, inv_perm, offsets, blk, wsplit, part, zpart, gpart, total;
 };
 LayerWs layer_ws(const ec2moe_layer_desc* d) {
   LayerWs w{};
@@ -257,6 +275,8 @@ LayerWs layer_ws(const ec2moe_layer_desc* d) {
   w.blk = take((size_t)route_blocks((long long)T * k) * d->E * 4);
   w.wsplit = take(gate_split_bytes(d->E, d->n_groups, d->d, is_bf16(d)));
   w.part = take(splitk_possible(d) ? (size_t)SPLITK_MAX * T * k * dm * 4 : 0);
+  w.zpart = take(is_bf16(d) && d->r > 0 && d->T <= 256 ? (size_t)ENC_SPLIT_MAX * T * d->r * 4 : 0);
+  w.gpart = take(gate_partial_bytes(d->T, d->d, d->E, d->n_groups));
   w.total = off;
   return w;
 }
@@ -357,7 +377,7 @@ struct RelPlace {  // relative placement of decoded rows (routing fused into the
 
 cudaError_t run_codec(const ec2moe_layer_desc* d, bool encode, const void* in, const void* V, void* out,
                       cudaStream_t s, const int32_t* inv_perm = nullptr, long long self_row_base = -1,
-                      const RelPlace& rel = RelPlace()) {
+                      const RelPlace& rel = RelPlace(), float* enc_partial = nullptr) {
   GemmArgs g = gemm_base();
   g.name = encode ? "lr_encode" : "lr_decode";
   g.A = in;
@@ -382,6 +402,15 @@ cudaError_t run_codec(const ec2moe_layer_desc* d, bool encode, const void* in, c
     g.rep_offsets_out = rel.offsets_out;
     g.rep_E = d->E;
     return run_gemm(d, g, EPI_REPLICATE, s);
+  }
+  const int split = encode && enc_partial ? enc_split(d) : 1;
+  if (split > 1) {
+    g.split_k = split;
+    g.partial = enc_partial;
+    g.part_rows = d->T;
+    cudaError_t e = run_gemm(d, g, EPI_PARTIAL, s);
+    if (e != cudaSuccess) return e;
+    return launch_splitk_sum(enc_partial, split, d->T, d->r, out, s);
   }
   return run_gemm(d, g, EPI_STORE, s);
 }
@@ -722,6 +751,8 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
     ga.route_rel = inv_perm;
     if (gate_split_bytes(desc->E, desc->n_groups, desc->d, bf)) ga.w_split = ws + L.wsplit;
   }
+  if (gate_partial_bytes(desc->T, desc->d, desc->E, desc->n_groups))
+    ga.gate_partial = reinterpret_cast<float*>(ws + L.gpart);
   bool routed = false;
   int gate_sms = 0;
   EC2MOE_CUDA(launch_gate(ga, bf, stream, &routed, &gate_sms));
@@ -762,7 +793,8 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
     ca.busy_sms = gate_sms;
     EC2MOE_CUDA(launch_codec_fused(ca, stream));
   } else if (desc->r > 0) {
-    EC2MOE_CUDA(run_codec(desc, true, X, w->V_enc, zbuf, stream));
+    EC2MOE_CUDA(run_codec(desc, true, X, w->V_enc, zbuf, stream, nullptr, -1, RelPlace(),
+                          reinterpret_cast<float*>(ws + L.zpart)));
     EC2MOE_CUDA(run_codec(desc, false, zbuf, w->V_dec, xa, stream, inv_perm, desc->n_shared > 0 ? n : -1, rel));
   } else {
     // Step 3b (move): rows of X into expert order; shared experts read X itself.
@@ -884,10 +916,13 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
       ga.route_rel = inv_perm;
       if (gate_split_bytes(sub.E, sub.n_groups, sub.d, bf)) ga.w_split = ws + L.wsplit;
     }
+    if (gate_partial_bytes(sub.T, sub.d, sub.E, sub.n_groups)) ga.gate_partial = reinterpret_cast<float*>(ws + L.gpart);
     bool routed = false;
     EC2MOE_CUDA(launch_gate(ga, bf, se, &routed));
     if (!routed) EC2MOE_CUDA(launch_route(idx_i, n, sub.E, blk, cnt_i, offsets, perm, inv_perm, se));
-    if (sub.r > 0) EC2MOE_CUDA(run_codec(&sub, true, Xi, w->V_enc, zbuf, se));
+    if (sub.r > 0)
+      EC2MOE_CUDA(run_codec(&sub, true, Xi, w->V_enc, zbuf, se, nullptr, -1, RelPlace(),
+                            reinterpret_cast<float*>(ws + L.zpart)));
     EC2MOE_CUDA(cudaEventRecord(events[1 + i], se));
 
     // ---- cloud: decoder into expert order, experts, combine

@@ -669,6 +669,178 @@ __global__ void __launch_bounds__(SL_THREADS) gate_tiled_kernel(const KParams p)
   }
 }
 
+// ---- small batches (T <= 256): the d_model axis split across CTAs
+// One or two 128-token tiles leave a per-tile kernel with one or two CTAs
+// walking all of d_model.  Here CTA (c, b) takes the GP_DC columns of chunk c
+// for the GP_TB tokens of tile b: it stages the gate-row slice (fp32) and the
+// activation slice (as fp32) in shared memory and writes the fp32 partial
+// logits of its chunk; a second kernel adds the chunks in chunk order, adds
+// the bias, and takes the same warp decision and in-kernel routing as the
+// other gates.  Partials: [n_chunks][T][O].
+constexpr int GP_TB = 64;
+constexpr int GP_DC = 128;
+constexpr int GP_PITCH = GP_DC + 4;  // floats; rows 16-byte aligned, float4 reads of 8 rows on distinct banks
+constexpr int GP_OB = 8;
+constexpr int GP_THREADS = 256;
+constexpr int GD_BT = 8;             // tokens per CTA of the decision kernel (one warp each)
+
+size_t gp_smem(int O) { return (size_t)(O + GP_TB) * GP_PITCH * sizeof(float); }
+
+template <typename TX>
+__global__ void __launch_bounds__(GP_THREADS) gate_partial_kernel(const KParams p, float* __restrict__ part) {
+  extern __shared__ float4 gp_smem_v[];
+  float* sW = reinterpret_cast<float*>(gp_smem_v);  // [O][GP_PITCH]
+  const int O = p.E + (p.K == 1 ? 0 : p.K);
+  float* sX = sW + (size_t)O * GP_PITCH;            // [GP_TB][GP_PITCH]
+  const int c0 = blockIdx.x * GP_DC;
+  const int t0 = blockIdx.y * GP_TB;
+  pdl_trigger();
+  // gate-row slice: constant weights, staged before waiting on the previous kernel
+  for (int i = threadIdx.x; i < O * (GP_DC / 4); i += GP_THREADS) {
+    const int o = i / (GP_DC / 4), c = (i % (GP_DC / 4)) * 4;
+    float4 v = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    if (c0 + c < p.d) {
+      const float* row = o < p.E ? p.W_local + (size_t)o * p.d : p.W_global + (size_t)(o - p.E) * p.d;
+      v = *reinterpret_cast<const float4*>(row + c0 + c);
+    }
+    *reinterpret_cast<float4*>(sW + o * GP_PITCH + c) = v;
+  }
+  pdl_wait();
+  if (p.route_counts && blockIdx.x == 0 && blockIdx.y == 0)
+    for (int e = threadIdx.x; e < p.E; e += GP_THREADS) p.route_counts[e] = 0;
+  const TX* X = reinterpret_cast<const TX*>(p.X);
+  for (int i = threadIdx.x; i < GP_TB * (GP_DC / 8); i += GP_THREADS) {
+    const int t = i / (GP_DC / 8), c = (i % (GP_DC / 8)) * 8;
+    float f[8];
+    Chunk8<TX> x;
+    if (t0 + t < p.T && c0 + c < p.d) x.load(X + (size_t)(t0 + t) * p.d + c0 + c);
+    else x.zero();
+    x.to_float(f);
+    *reinterpret_cast<float4*>(sX + t * GP_PITCH + c) = make_float4(f[0], f[1], f[2], f[3]);
+    *reinterpret_cast<float4*>(sX + t * GP_PITCH + c + 4) = make_float4(f[4], f[5], f[6], f[7]);
+  }
+  __syncthreads();
+  // item = (token t, block of GP_OB gate rows); lanes run over tokens so the
+  // gate-row reads are warp broadcasts
+  const int nob = (O + GP_OB - 1) / GP_OB;
+  for (int item = threadIdx.x; item < GP_TB * nob; item += GP_THREADS) {
+    const int t = item % GP_TB, ob = item / GP_TB;
+    const int tok = t0 + t;
+    if (tok >= p.T) continue;
+    float acc[GP_OB];
+#pragma unroll
+    for (int j = 0; j < GP_OB; ++j) acc[j] = 0.0f;
+    const float* xr = sX + t * GP_PITCH;
+#pragma unroll 4
+    for (int c = 0; c < GP_DC; c += 4) {
+      const float4 xv = *reinterpret_cast<const float4*>(xr + c);
+#pragma unroll
+      for (int j = 0; j < GP_OB; ++j) {
+        const int o = ob * GP_OB + j < O ? ob * GP_OB + j : O - 1;  // clamped read, result unused
+        const float4 wv = *reinterpret_cast<const float4*>(sW + o * GP_PITCH + c);
+        acc[j] = fmaf(xv.x, wv.x, acc[j]);
+        acc[j] = fmaf(xv.y, wv.y, acc[j]);
+        acc[j] = fmaf(xv.z, wv.z, acc[j]);
+        acc[j] = fmaf(xv.w, wv.w, acc[j]);
+      }
+    }
+    float* dst = part + ((size_t)blockIdx.x * p.T + tok) * O;
+#pragma unroll
+    for (int j = 0; j < GP_OB; ++j)
+      if (ob * GP_OB + j < O) dst[ob * GP_OB + j] = acc[j];
+  }
+}
+
+// Decision kernel: GD_BT tokens per CTA (one warp each).  The chunk sums are
+// split four ways (group g adds chunks g, g + 4, ... in order; then the four
+// group sums are added in group order), so each thread keeps eight loads in
+// flight and the result does not depend on the launch.
+constexpr int GD_SPLIT = 4;
+__global__ void __launch_bounds__(SL_THREADS) gate_decide_kernel(const KParams p, const float* __restrict__ part,
+                                                                 int n_chunks) {
+  extern __shared__ float4 gd_smem_v[];
+  const int O = p.E + (p.K == 1 ? 0 : p.K);
+  const int pairs = GD_BT * O;
+  float* sLog = reinterpret_cast<float*>(gd_smem_v);                  // [GD_BT][O]
+  float* sGrp = sLog + pairs;                                          // [GD_SPLIT][GD_BT * O]
+  int* sIdx = reinterpret_cast<int*>(sGrp + GD_SPLIT * pairs);        // [GD_BT * k]
+  __shared__ int s_base[128];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int tile = blockIdx.x;
+  pdl_trigger();
+  pdl_wait();
+  const size_t plane = (size_t)p.T * O;
+  for (int i = threadIdx.x; i < GD_SPLIT * pairs; i += SL_THREADS) {
+    const int g = i / pairs, pr = i % pairs;
+    const int tok = tile * GD_BT + pr / O;
+    float sum = 0.0f;
+    if (tok < p.T) {
+      const float* src = part + (size_t)tok * O + pr % O;
+      for (int c0 = g; c0 < n_chunks; c0 += 8 * GD_SPLIT) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int c = c0 + u * GD_SPLIT;
+          v[u] = c < n_chunks ? src[(size_t)c * plane] : 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) sum += v[u];  // chunk order within the group
+      }
+    }
+    sGrp[i] = sum;
+  }
+  __syncthreads();
+  for (int pr = threadIdx.x; pr < pairs; pr += SL_THREADS) {
+    const int o = pr % O;
+    float sum = sGrp[pr];
+#pragma unroll
+    for (int g = 1; g < GD_SPLIT; ++g) sum += sGrp[g * pairs + pr];
+    sLog[pr] = sum + (o < p.E ? p.b_local[o] : p.b_global[o - p.E]);
+  }
+  __syncthreads();
+  for (int jj = warp; jj < GD_BT; jj += SL_THREADS / 32) {
+    const int tok = tile * GD_BT + jj;
+    if (tok < p.T) decide_token_warp(p, sLog + jj * O, tok, lane, p.route_counts ? sIdx + jj * p.k : nullptr);
+  }
+  __syncthreads();
+  if (p.route_counts) route_tile(p, tile, GD_BT, sIdx, s_base);
+}
+
+constexpr int GP_MAX_T = 256;
+constexpr int GP_MIN_D = 1024;
+
+}  // namespace
+
+size_t gate_partial_bytes(int T, int d, int E, int K) {
+  const int O = E + (K == 1 ? 0 : K);
+  if (T < 1 || T > GP_MAX_T || d < GP_MIN_D || d % 8 != 0 || O > MAXO) return 0;
+  return (size_t)((d + GP_DC - 1) / GP_DC) * T * O * sizeof(float);
+}
+
+namespace {
+
+template <typename TX>
+cudaError_t launch_gate_partial(const GateArgs& a, const KParams& p, int O, cudaStream_t s) {
+  const int n_chunks = (a.d + GP_DC - 1) / GP_DC;
+  const int smem_a = static_cast<int>(gp_smem(O));
+  cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(gate_partial_kernel<TX>), smem_a);
+  if (e != cudaSuccess) return e;
+  {
+    KernelScope ks("gate_topk", s);
+    e = launch_kernel(gate_partial_kernel<TX>, dim3(n_chunks, (a.T + GP_TB - 1) / GP_TB), dim3(GP_THREADS),
+                      (size_t)smem_a, s, p, a.gate_partial);
+    if (e != cudaSuccess) return e;
+  }
+  const int smem_b = (GD_BT * O * (1 + GD_SPLIT) + GD_BT * a.k) * 4;
+  e = ensure_smem_attr(reinterpret_cast<const void*>(gate_decide_kernel), smem_b);
+  if (e != cudaSuccess) return e;
+  KernelScope ks("gate_decide", s);
+  e = launch_kernel(gate_decide_kernel, dim3((a.T + GD_BT - 1) / GD_BT), dim3(SL_THREADS), (size_t)smem_b, s, p,
+                    static_cast<const float*>(a.gate_partial), n_chunks);
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* routed, int* held_sms) {
@@ -695,6 +867,17 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* rout
   p.route_rel = nullptr;
   const int O = a.E + (a.K == 1 ? 0 : a.K);
   cudaError_t e;
+  if (a.gate_partial && gate_partial_bytes(a.T, a.d, a.E, a.K) &&
+      reinterpret_cast<uintptr_t>(a.gate_partial) % 16 == 0 && reinterpret_cast<uintptr_t>(a.W_local) % 16 == 0 &&
+      (a.K == 1 || reinterpret_cast<uintptr_t>(a.W_global) % 16 == 0)) {
+    if (a.route_counts && a.route_rel) {
+      p.route_counts = a.route_counts;
+      p.route_rel = a.route_rel;
+      if (routed) *routed = true;
+    }
+    if (held_sms) *held_sms = (a.T + GD_BT - 1) / GD_BT;
+    return bf16 ? launch_gate_partial<__nv_bfloat16>(a, p, O, s) : launch_gate_partial<float>(a, p, O, s);
+  }
   {
     bool handled = false;
     e = launch_gate_tensor(a, p, O, bf16, s, routed, held_sms, &handled);

@@ -83,9 +83,15 @@ struct GateArgs {
   // terms by a small kernel launched first; nullptr: the gate kernel splits
   // them itself.
   void* w_split;
+  // Optional workspace of gate_partial_bytes() bytes (16-byte aligned): small
+  // batches then split d_model across CTAs (partial logits, then a decision
+  // kernel); nullptr: the per-tile gates.
+  float* gate_partial;
 };
 // Bytes of the prepared split gate rows (0 when the tensor-core gate does not apply).
 size_t gate_split_bytes(int E, int K, int d, bool bf16);
+// Bytes of the small-batch gate's partial logits (0 when that gate does not apply).
+size_t gate_partial_bytes(int T, int d, int E, int K);
 // Launches the gate; with the routing fields set, also fills them when the
 // fused path applies (*routed = true), else gate only.  *held_sms (optional)
 // receives how many SMs the gate kernel's CTAs occupy while it runs.
@@ -114,6 +120,9 @@ cudaError_t launch_gather(const void* src, void* dst, const int32_t* perm, long 
                           bool bf16, cudaStream_t s);
 // counts[e] = sum_p parts[p*E + e], p ascending.
 cudaError_t launch_sum_counts(const int32_t* parts, int n_parts, int E, int32_t* counts, cudaStream_t s);
+// out[row][c] = bf16(partial[0][row][c] + ... + partial[S-1][row][c]) for
+// rows < `rows`, c < N (N % 4 == 0): the split-K encoder's reduce.
+cudaError_t launch_splitk_sum(const float* partial, int S, long long rows, int N, void* out, cudaStream_t s);
 // Split-K expert output: y[t] = sum_slot w[t*k+slot] * sum_s partial[s][pos(t, slot)]
 // + sum_j shared[j*T+t], with pos = offsets[idx[i]] + rel[i] (rel_mode) or rel[i].
 cudaError_t launch_splitk_combine(const float* partial, int split_k, long long part_rows, const int32_t* offsets,

@@ -366,6 +366,76 @@ cudaError_t launch_sum_counts(const int32_t* parts, int n_parts, int E, int32_t*
   return cudaGetLastError();
 }
 
+// Split-K sums into bf16.  A block covers 64 (row, 4-column) items with 4
+// threads each: thread group g adds the planes s = g, g + 4, ... (8 loads in
+// flight), then the four group sums are added in group order and rounded
+// once -- a fixed order, so the result does not depend on the launch.
+constexpr int SUM_ITEMS = 64;
+constexpr int SUM_GROUPS = 4;
+__global__ void __launch_bounds__(SUM_ITEMS * SUM_GROUPS)
+    splitk_sum_kernel(const float* __restrict__ partial, int S, long long rows, int N,
+                      __nv_bfloat16* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float4 part[SUM_GROUPS][SUM_ITEMS];
+  const int it = threadIdx.x % SUM_ITEMS, grp = threadIdx.x / SUM_ITEMS;
+  const long long per_row = N / 4;
+  const long long total = rows * per_row;
+  const long long plane = rows * N;
+  for (long long base = (long long)blockIdx.x * SUM_ITEMS; base < total; base += (long long)gridDim.x * SUM_ITEMS) {
+    const long long i = base + it;
+    const long long at = i < total ? (i / per_row) * N + (i % per_row) * 4 : 0;
+    float4 acc = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    if (i < total) {
+      for (int s0 = grp; s0 < S; s0 += 8 * SUM_GROUPS) {
+        float4 v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int s = s0 + j * SUM_GROUPS;
+          v[j] = s < S ? *reinterpret_cast<const float4*>(partial + s * plane + at) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          acc.x += v[j].x;
+          acc.y += v[j].y;
+          acc.z += v[j].z;
+          acc.w += v[j].w;
+        }
+      }
+    }
+    part[grp][it] = acc;
+    __syncthreads();
+    if (grp == 0 && i < total) {
+      float4 t = part[0][it];
+#pragma unroll
+      for (int g = 1; g < SUM_GROUPS; ++g) {
+        t.x += part[g][it].x;
+        t.y += part[g][it].y;
+        t.z += part[g][it].z;
+        t.w += part[g][it].w;
+      }
+      uint2 o;
+      o.x = pack_bf16x2(t.x, t.y);
+      o.y = pack_bf16x2(t.z, t.w);
+      *reinterpret_cast<uint2*>(out + at) = o;
+    }
+    __syncthreads();
+  }
+}
+
+cudaError_t launch_splitk_sum(const float* partial, int S, long long rows, int N, void* out, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  const long long total = rows * (N / 4);
+  long long blocks = (total + SUM_ITEMS - 1) / SUM_ITEMS;
+  const long long cap = (long long)sm_count() * 8;
+  if (blocks > cap) blocks = cap;
+  KernelScope ks("lr_reduce", s);
+  cudaError_t e = launch_kernel(splitk_sum_kernel, dim3(static_cast<int>(blocks)), dim3(SUM_ITEMS * SUM_GROUPS), 0, s,
+                                partial, S, rows, N, static_cast<__nv_bfloat16*>(out));
+  if (e != cudaSuccess) return e;
+  return cudaGetLastError();
+}
+
 // Split-K expert outputs (bf16 layers): for every token and 8-column chunk,
 // the k slots' fp32 partial sums over the K ranges are added (range order),
 // weighted by the slot's gate weight (slot order), plus the shared experts'

@@ -92,12 +92,17 @@ def rel_fro(a: np.ndarray, b: np.ndarray) -> float:
     return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-300))
 
 
-def output_check(y_gpu: np.ndarray, y_ref: np.ndarray, bf16: bool):
+def output_check(y_gpu: np.ndarray, y_ref: np.ndarray, bf16: bool, pair: bool = False):
+    """The output tolerances against the oracle.  pair=True compares two GPU
+    outputs that take different rounding paths: each lies within the bound of
+    the exact result, so their difference is held to twice the max-abs bound
+    (the Frobenius bound stays)."""
     err = rel_fro(y_gpu, y_ref)
     mx = float(np.abs(y_gpu - y_ref).max()) if y_ref.size else 0.0
     if bf16:
+        mx_bound = 6e-2 if pair else 3e-2
         assert err <= 1e-2, f"relative Frobenius error {err:.3e} > 1e-2"
-        assert mx <= 3e-2, f"max abs error {mx:.3e} > 3e-2"
+        assert mx <= mx_bound, f"max abs error {mx:.3e} > {mx_bound:.0e}"
     else:
         assert err <= 1e-4, f"relative Frobenius error {err:.3e} > 1e-4"
     return err, mx

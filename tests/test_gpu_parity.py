@@ -116,6 +116,25 @@ def test_gate_nonfinite_token_names_valid_experts(cfg):
     assert n_excl <= 2, n_excl
 
 
+@pytest.mark.parametrize("cfg", [S.preset("decode_bf16", T=16, n_allowed=4, seed=25),
+                                 S.preset("finegrained_bf16", T=40, seed=26)], ids=lambda c: f"{c.name}-T{c.T}")
+def test_layer_nonfinite_token_small_batch(cfg):
+    """The small-batch gate of the layer path (d_model split across CTAs) takes
+    the same decision for a NaN token: the k lowest allowed experts; its routing
+    tables stay consistent."""
+    inp = S.make_inputs(cfg, device="cuda")
+    bad = [0, cfg.T - 1]
+    inp["X"][bad] = float("nan")
+    run = LayerRun(cfg, inp)
+    run.forward()
+    torch.cuda.synchronize()
+    gi = run.topk_idx.cpu().numpy()
+    allowed = np.flatnonzero(inp["mask"].cpu().numpy())
+    for t in bad:
+        assert sorted(gi[t].tolist()) == allowed[: cfg.k].tolist()
+    assert np.array_equal(run.counts.cpu().numpy(), np.bincount(gi.ravel(), minlength=cfg.E))
+
+
 ROUTE_CASES = [S.preset("tiny_fp32"), S.preset("switch_bf16"), S.preset("finegrained_bf16"),
                S.preset("switch_bf16", T=1000, k=2, seed=9), S.preset("decode_bf16", T=1, seed=1)]
 
@@ -195,6 +214,14 @@ LAYER_CASES = [
     (S.preset("switch_bf16", T=2, seed=43), None),
     (S.preset("decode_bf16", T=1, n_allowed=8, r=256, seed=46), None),
     (S.preset("mixtral_bf16", T=3, seed=44), None),
+    # split-K encoder with a K range count the k-block count does not divide
+    # (33 k-blocks of 64 in 11 ranges of 3)
+    (S.preset("decode_bf16", T=7, d=2112, d_ff=2048, n_allowed=8, r=256, seed=49), None),
+    # small batches with d_model split across the gate's CTAs: group gate
+    # with several token tiles, 72 gate rows, and an fp32 layer
+    (S.preset("mixtral_bf16", T=129, seed=50), None),
+    (S.preset("finegrained_bf16", T=200, seed=51), None),
+    (S.preset("tiny_fp32", T=100, d=1024, seed=52), None),
     (S.preset("tiny_fp32", T=7, seed=45), None),
     # the limits: 128 experts in 16 groups, Top-8, 144 gate rows; and many
     # tiles per CTA in every kernel
