@@ -104,7 +104,16 @@ struct Cfg {
   static constexpr int TMEM_COLS = pow2_at_least(2 * BN);  // two accumulators
   static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8;
   static constexpr int STG_PITCH = CW * 2 + 16;          // bytes per staged row (padded)
-  static constexpr int STG_BYTES = EPI_WARPS * 32 * STG_PITCH;
+  // Row-segment epilogue (contiguous or per-row destinations): the four warps
+  // of a lane quadrant stage 32 rows x 64 columns (bf16, 128-byte rows,
+  // 16-byte chunks XOR-swizzled by row) and store whole 128-byte row
+  // segments.  EPI_REPLICATE keeps per-warp 32 x 16 chunks; EPI_PARTIAL
+  // writes fp32 from registers.
+  static constexpr bool ROWSEG =
+      (EPI == EPI_STORE || EPI == EPI_GELU || EPI == EPI_SWIGLU || EPI == EPI_SCATTER) && BN_OUT % 64 == 0;
+  static constexpr int SLAB = 64;
+  static constexpr int STG_BYTES =
+      ROWSEG ? 4 * 32 * SLAB * 2 : (EPI == EPI_PARTIAL ? 0 : EPI_WARPS * 32 * STG_PITCH);
   static constexpr int OFF_INTS = 132;  // expert offsets of EPI_REPLICATE's relative mode (<= 128 + 1, padded)
   static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES + 16 + 2 * (MAX_GROUPS + 1) * 4 + OFF_INTS * 4 +
                               STG_BYTES;
@@ -337,9 +346,69 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
       }
-      if (!mbar_wait(smem_u32(&tfull[acc]), acc_phase, budget, abort_flag, &g_tc_error)) break;
+      bool ok = mbar_wait(smem_u32(&tfull[acc]), acc_phase, budget, abort_flag, &g_tc_error);
+      if (C::ROWSEG) {
+        // the quadrant's four warps take the same path (they meet at named barriers)
+        uint32_t all_ok;
+        asm volatile(
+            "{\n .reg .pred p, r;\n setp.ne.u32 p, %1, 0;\n"
+            " bar.red.and.pred r, %2, 128, p;\n selp.u32 %0, 1, 0, r;\n}"
+            : "=r"(all_ok)
+            : "r"(ok ? 1u : 0u), "r"(1 + q)
+            : "memory");
+        ok = all_ok != 0;
+      }
+      if (!ok) break;
       tc_fence_after();
       const uint32_t t_row = tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(q * 32) << 16);
+      if constexpr (C::ROWSEG) {
+        // Slabs of 64 output columns: warp `part` rounds its 16 columns of the
+        // slab for the quadrant's 32 rows into the quadrant's staging slab,
+        // then each warp stores 8 of the 32 rows as 128-byte row segments (4
+        // rows per store instruction).  The destination row of staged row rr
+        // comes from lane rr, which owns that row in every warp of the quadrant.
+        uint8_t* slab = stg_all + q * (32 * C::SLAB * 2);
+        constexpr int NSLAB = C::BN_OUT / C::SLAB;
+#pragma unroll 1
+        for (int sl = 0; sl < NSLAB; ++sl) {
+          const int c0 = sl * C::SLAB + part * 16;
+          uint32_t rv[16], ru[16];
+          tmem_ld_nw<16>(t_row + c0, rv);
+          if (EPI == EPI_SWIGLU) tmem_ld_nw<16>(t_row + c0 + BN / 2, ru);
+          tmem_wait();
+          float v[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            v[i] = __uint_as_float(rv[i]);
+            if (EPI == EPI_SWIGLU) v[i] = silu_bf16out(v[i]) * __uint_as_float(ru[i]);
+            else if (EPI == EPI_GELU) v[i] = gelu_bf16out(v[i]);
+            else if (EPI == EPI_SCATTER) v[i] *= sc;
+          }
+#pragma unroll
+          for (int j = 0; j < 2; ++j) {
+            U4 q4{pack_bf16x2(v[8 * j + 0], v[8 * j + 1]), pack_bf16x2(v[8 * j + 2], v[8 * j + 3]),
+                  pack_bf16x2(v[8 * j + 4], v[8 * j + 5]), pack_bf16x2(v[8 * j + 6], v[8 * j + 7])};
+            *reinterpret_cast<U4*>(slab + lane * 128 + (((2 * part + j) ^ (lane & 7)) * 16)) = q4;
+          }
+          asm volatile("bar.sync %0, 128;" ::"r"(1 + q) : "memory");
+          const int seg = lane & 7;
+          const int col = tc.n_blk * C::BN_OUT + sl * C::SLAB + seg * 8;
+#pragma unroll
+          for (int pass = 0; pass < 2; ++pass) {
+            const int rr = part * 8 + pass * 4 + (lane >> 3);
+            const bool rvalid = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr) != 0;
+            const long long drow = __shfl_sync(0xffffffffu, dest, rr);
+            const U4 q4 = *reinterpret_cast<const U4*>(slab + rr * 128 + ((seg ^ (rr & 7)) * 16));
+            if (rvalid && col < p.N)
+              *reinterpret_cast<U4*>(reinterpret_cast<__nv_bfloat16*>(p.out) + drow * p.ldo + col) = q4;
+          }
+          asm volatile("bar.sync %0, 128;" ::"r"(1 + q) : "memory");
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+        continue;
+      }
       // Each chunk of 32 rows x CW columns is staged in shared memory (thread =
       // row) and written back with CW/8 lanes per row, so a warp store writes
       // whole 32-byte sectors of 16 rows instead of 16-byte pieces of 32 rows.
