@@ -107,6 +107,21 @@ def test_workspace_sizes(lib):
     assert C.ec2moe_workspace_size(_desc(E=9)) == 0
 
 
+def test_workspace_covers_decode_regions(lib):
+    """Decode-sized bf16 calls add fp32 partial-sum regions: the small-batch
+    gate's [d/128, T, E+K] logits, the split-K encoder's [<=32, T, r] and the
+    split-K down projection's [<=8, T*k, d]; larger batches add none of them."""
+    T, d, E, K, k, r, ff = 64, 4096, 8, 2, 2, 256, 14336
+    ws = C.ec2moe_workspace_size(_desc(T=T, d=d, E=E, n_groups=K, k=k, r=r, d_ff=ff))
+    es = 2
+    dense = (T * r + (T * k + T) * d + T * k * ff + T * k * d) * es
+    partials = (d // 128) * T * (E + K) * 4 + 32 * T * r * 4 + 8 * T * k * d * 4
+    assert ws >= dense + partials
+    big = C.ec2moe_workspace_size(_desc(T=300, d=d, E=E, n_groups=K, k=k, r=r, d_ff=ff))
+    big_dense = (300 * r + (300 * k + 300) * d + 300 * k * ff + 300 * k * d) * es
+    assert big_dense <= big < big_dense + 4 * 1024 * 1024  # no T-sized partial regions
+
+
 def test_other_entry_points_validate(lib):
     A = 0x100000
     d = _desc()
