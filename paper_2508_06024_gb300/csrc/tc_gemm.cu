@@ -12,9 +12,12 @@
 // CTA layout (576 threads):
 //   warp 0      TMA producer (one elected lane)
 //   warp 1      TMEM allocator + MMA issuer (one elected lane)
-//   warps 2..17 epilogue: TMEM -> registers -> global.  Warp w may only read
-//               TMEM lanes 32*(w%4) .. +31 (rows of the 128-row tile); the
-//               four warps of a lane quadrant split the tile's columns.
+//   warps 2..17 epilogue: TMEM -> registers -> shared staging -> global.
+//               Warp w may only read TMEM lanes 32*(w%4) .. +31 (rows of the
+//               128-row tile); the four warps of a lane quadrant split the
+//               tile's columns and, for contiguous or per-row destinations,
+//               stage 64-column slabs together (named barrier per quadrant)
+//               to store whole 128-byte row segments.
 // Pipelines: STAGES shared-memory stages (full/empty mbarriers) and two TMEM
 // accumulators (tmem_full/tmem_empty) so the epilogue of tile i overlaps the
 // main loop of tile i+1.
@@ -22,7 +25,9 @@
 // Every mbarrier wait is bounded by a clock64 budget.  A wait that gives up
 // sets the device error word, raises a CTA-wide abort flag that ends every
 // other wait at once, waits (again bounded) for the CTA's own TMA copies and
-// MMAs still in flight, frees TMEM and returns.
+// MMAs still in flight, frees TMEM and returns.  The warps of a quadrant agree
+// on the outcome of their accumulator wait (bar.red.and) before they meet at
+// their named barriers, so a timeout never leaves one of them behind.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
