@@ -115,7 +115,10 @@ typedef struct ec2moe_layer_weights {
 /* Bytes of device workspace ec2moe_layer_forward needs for `desc` (0 on an
  * invalid desc).  The workspace holds the codec output Z, the decoded and
  * expert-ordered activations, the expert hidden activations, per-slot expert
- * outputs and the routing tables. */
+ * outputs, the routing tables and the prepared gate rows; for decode-sized
+ * bf16 calls (T <= 256) also the fp32 partial sums of the split-d_model gate,
+ * the split-K encoder and the split-K down projection.  Its contents need no
+ * initialisation and are not preserved between calls. */
 size_t ec2moe_workspace_size(const ec2moe_layer_desc* desc);
 
 /* Bytes of device workspace ec2moe_experts needs (hidden activations). */
