@@ -23,7 +23,8 @@ GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "wor
 
 def _num(v):
     if isinstance(v, str):
-        return {"ln2": math.log(2.0), "ln3": math.log(3.0), "ln3-0.5": math.log(3.0) - 0.5}[v]
+        return {"ln2": math.log(2.0), "ln3": math.log(3.0), "ln4": math.log(4.0), "ln5": math.log(5.0),
+                "ln3-0.5": math.log(3.0) - 0.5}[v]
     return float(v)
 
 
@@ -374,6 +375,35 @@ def pin_layer_codec_golden(orc):
     assert out["idx"][:, 0].tolist() == [1, 1]
 
 
+def pin_layer_pairing_golden(orc):
+    """Eq. 1 pairs G(x)_i with E_i(x): three distinct experts, Top-2 with unequal
+    weights, two tokens routed to different expert pairs, and the hand-derived
+    y of each (GELU, GELU with renormalised weights, SwiGLU).  A routed row that
+    met another expert's weights, or a slot scaled by another slot's weight,
+    changes y here."""
+    ex = golden()["layer_pairing"]
+    X = np.array(ex["x"])
+    W1, W3, W2 = (np.array(ex[key]) for key in ("W1", "W3", "W2"))
+    base = dict(X=X, W_local=np.array([[_num(v) for v in row] for row in ex["W_local"]]),
+                b_local=np.array(ex["b_local"]), W_global=None, b_global=None,
+                mask=np.array(ex["mask"], np.uint8), W1=W1, W3=None, W2=W2, W1s=None, W3s=None, W2s=None,
+                V_enc=None, V_dec=None)
+    for act, renorm, key in [(orc.GELU, False, "y_gelu"), (orc.GELU, True, "y_gelu_renorm"),
+                             (orc.SWIGLU, False, "y_swiglu")]:
+        inp = dict(base, W3=W3 if act == orc.SWIGLU else None)
+        out = orc.layer_forward(inp, ex["n_groups"], ex["k"], act, renorm=renorm)
+        assert out["idx"].tolist() == ex["idx"]
+        w = np.array(ex["w"])
+        if renorm:
+            w = w / w.sum(axis=1, keepdims=True)
+        np.testing.assert_allclose(out["w"], w, rtol=0, atol=1e-15)
+        np.testing.assert_allclose(out["y"], ex[key], rtol=0, atol=1e-14)
+        # each token row alone gives the same row (rows are independent)
+        for t in range(2):
+            part = orc.layer_forward(inp, ex["n_groups"], ex["k"], act, renorm=renorm, rows=[t])
+            np.testing.assert_allclose(part["y"][0], ex[key][t], rtol=0, atol=1e-14)
+
+
 def pin_layer_rows_subset(orc, seed=13):
     """Computing the expert part on a subset of rows gives those rows of the full result
     (tokens are independent in Eq. 1)."""
@@ -391,5 +421,5 @@ ALL_PINS = [
     pin_group_factorisation, pin_topk_bruteforce, pin_rejections, pin_route_golden,
     pin_route_invariants, pin_codec_golden, pin_codec_identity, pin_codec_projection,
     pin_ffn_golden, pin_activations_library, pin_ffn_bruteforce, pin_layer_single_expert,
-    pin_layer_linearity, pin_layer_codec_golden, pin_layer_rows_subset,
+    pin_layer_linearity, pin_layer_codec_golden, pin_layer_rows_subset, pin_layer_pairing_golden,
 ]

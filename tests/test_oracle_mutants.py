@@ -127,6 +127,43 @@ def m_experts_see_raw_x(inp, n_groups, k, act, renorm=False, rows=None):
     return out
 
 
+def m_experts_rolled(inp, n_groups, k, act, renorm=False, rows=None):
+    # every routed row meets the weights of expert e - 1 instead of expert e
+    inp = dict(inp)
+    for key in ("W1", "W3", "W2"):
+        if inp.get(key) is not None:
+            inp[key] = np.roll(np.asarray(inp[key]), 1, axis=0)
+    return _layer_forward(inp, n_groups, k, act, renorm, rows)
+
+
+def m_slot_weight_shifted(inp, n_groups, k, act, renorm=False, rows=None):
+    # slot s's expert output is scaled by slot s + 1's gate weight
+    out = _layer_forward(inp, n_groups, k, act, renorm, rows)
+    X_hat = out["X_hat"]
+    sel = out["rows"]
+    idx, w = out["idx"][sel], out["w"][sel]
+    y = np.zeros_like(out["y"])
+    for e in range(inp["W1"].shape[0]):
+        for s in range(k):
+            hit = np.nonzero(idx[:, s] == e)[0]
+            if hit.size == 0:
+                continue
+            W3 = None if inp.get("W3") is None else inp["W3"][e]
+            o = orc.expert_ffn(X_hat[hit], inp["W1"][e], inp["W2"][e], W3, act)
+            y[hit] += w[hit, (s + 1) % k][:, None] * o
+    if inp.get("W1s") is not None:
+        for s in range(inp["W1s"].shape[0]):
+            W3s = None if inp.get("W3s") is None else inp["W3s"][s]
+            y += orc.expert_ffn(X_hat, inp["W1s"][s], inp["W2s"][s], W3s, act)
+    out["y"] = y
+    return out
+
+
+def m_weights_slot_rolled(g, idx, renorm):
+    # the combine weights are paired with the wrong slots
+    return np.roll(_combine_weights(g, idx, renorm), 1, axis=1)
+
+
 def m_gap_wrong_sign(log_g, idx, allowed):
     b, a = _topk_gaps(log_g, idx, allowed)
     return -b, a
@@ -150,6 +187,9 @@ MUTANTS = [
     ("combine_weights", m_renorm_always),
     ("layer_forward", m_no_shared),
     ("layer_forward", m_experts_see_raw_x),
+    ("layer_forward", m_experts_rolled),
+    ("layer_forward", m_slot_weight_shifted),
+    ("combine_weights", m_weights_slot_rolled),
     ("topk_gaps", m_gap_wrong_sign),
 ]
 
