@@ -4,9 +4,11 @@
 A step is one ``ec2moe_layer_forward`` (mask -> group gate -> Top-k ->
 histogram/permute -> low-rank encode/decode -> grouped expert FFN ->
 gate-weighted combine) over one batch of synthetic tokens of the workload.
-Default workload: the Switch-style bf16 layer (4096 tokens = batch 8 x seq 512,
-d_model 768, 16 GELU experts with d_ff 3072, Top-1, 12 of 16 experts allowed,
-rank-128 codec).
+Default workload: the Mixtral-shaped bf16 layer, the largest configuration
+that fits one GPU (8192 tokens, d_model 4096, 8 SwiGLU experts with d_ff
+14336, Top-2, 2 groups of 4, 6 of 8 experts allowed, rank-512 codec);
+``--workload switch_bf16`` / ``finegrained_bf16`` / ``decode_bf16`` select the
+others.
 
 Timing: W untimed warm-up steps, then K steps, each bracketed by CUDA events
 on the launching stream with L2 flushed (256 MiB write) between steps; a
@@ -14,9 +16,12 @@ barrier and a device synchronise bracket the timed loop; the max over ranks is
 reported.  ``value`` replays one ``ec2moe_layer_forward`` call captured in a
 CUDA graph (inputs resident in HBM); ``e2e`` calls the C ABI eagerly every step
 with the host<->device copies of X and y inside the timed region.  Per-kernel
-times come from CUDA events the library records around each of its launches
-(``ec2moe_profile_*``) inside a graph-captured call.  Under torchrun each rank runs its own batch (token-parallel
-replicas, no collective on the data path; weak scaling).
+times: for each launch index i of the call, a graph of the whole call in which
+the library brackets only launch i with a pair of CUDA events
+(``ec2moe_profile_only``), replayed with L2 flushed; the kernel's neighbours
+keep their programmatic overlap and no other event node sits in the step.
+Under torchrun each rank runs its own batch (token-parallel replicas, no
+collective on the data path; weak scaling).
 
 ``--impl reference`` times the fp64 CPU oracle instead, on the host cores.
 """
@@ -47,7 +52,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="switch_bf16")
+    ap.add_argument("--workload", default="mixtral_bf16")
     ap.add_argument("--T", type=int, default=0, help="override the token count (0 = preset)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--pipeline", type=int, default=0,
@@ -251,6 +256,63 @@ def whole_job_tokens_per_s(world: int, tokens_per_rank: int, max_ms_per_step: fl
 
 
 # ------------------------------------------------------------------ reference arm (fp64 oracle on CPU)
+def blas_threads():
+    """(threads, library) of the BLAS numpy uses, read from the loaded OpenBLAS
+    (or MKL) itself; (None, None) when it cannot be read."""
+    import ctypes
+    import numpy  # noqa: F401  (loads the BLAS)
+    try:
+        from threadpoolctl import threadpool_info
+        for d in threadpool_info():
+            if d.get("user_api") == "blas":
+                return int(d["num_threads"]), d.get("internal_api")
+    except Exception:
+        pass
+    try:
+        with open("/proc/self/maps") as f:
+            libs = sorted({ln.split()[-1] for ln in f if "openblas" in ln.lower() and ".so" in ln})
+    except OSError:
+        libs = []
+    for path in libs:
+        try:
+            lib = ctypes.CDLL(path)
+        except OSError:
+            continue
+        for sym in ("scipy_openblas_get_num_threads64_", "openblas_get_num_threads64_", "openblas_get_num_threads",
+                    "scipy_openblas_get_num_threads"):
+            fn = getattr(lib, sym, None)
+            if fn is not None:
+                fn.restype = ctypes.c_int
+                return int(fn()), "openblas"
+    return None, None
+
+
+def oracle_inputs_from(inp):
+    """float64 numpy views of stored tensors for the oracle; expert weights are
+    widened one expert at a time when the oracle touches them."""
+    from paper_2508_06024_gb300 import synth as S
+
+    class Lazy:
+        def __init__(self, t):
+            self.t = t
+            self.shape = tuple(t.shape)
+
+        def __getitem__(self, i):
+            return S.to_f64(self.t[i])
+
+    out = {}
+    for k, v in inp.items():
+        if v is None:
+            out[k] = None
+        elif k == "mask":
+            out[k] = v.to("cpu").numpy().astype("uint8")
+        elif k in ("W1", "W3", "W2", "W1s", "W3s", "W2s"):
+            out[k] = Lazy(v.to("cpu"))
+        else:
+            out[k] = S.to_f64(v)
+    return out
+
+
 def oracle_sample_step(cfg, o, rows):
     from oracle import ec2moe_oracle as orc
     sub = dict(o)
@@ -260,24 +322,31 @@ def oracle_sample_step(cfg, o, rows):
 
 def oracle_inputs_cpu(cfg):
     from paper_2508_06024_gb300 import synth as S
-    inp = S.make_inputs(cfg, device="cpu")
-    out = {}
-    for k, v in inp.items():
-        if v is None:
-            out[k] = None
-        elif k == "mask":
-            out[k] = v.numpy().astype("uint8")
-        else:
-            out[k] = S.to_f64(v)
-    return out
+    return oracle_inputs_from(S.make_inputs(cfg, device="cpu"))
 
 
-def time_oracle(cfg, budget_s: float, steps: int = 0):
-    """Tokens/s of the oracle on a bounded sample of the workload's tokens.
+def time_oracle(cfg, budget_s: float, steps: int = 0, inp=None):
+    """Tokens/s of the oracle on a bounded sample of the workload's tokens
+    (inputs: the given stored tensors, else drawn on the CPU).
 
-    Returns (tokens_per_s, sample_desc, per_step_seconds list)."""
+    Returns (tokens_per_s, sample_desc, per_step_seconds list, tokens per step)."""
     import numpy as np
-    o = oracle_inputs_cpu(cfg)
+    o = oracle_inputs_cpu(cfg) if inp is None else oracle_inputs_from(inp)
+    # widen the weights of the experts the oracle can touch (allowed routed
+    # experts, every shared one) before timing: input conversion is not oracle work
+    allowed = np.flatnonzero(o["mask"])
+
+    class Widened:
+        def __init__(self, lazy, which):
+            self.shape = lazy.shape
+            self.rows = {int(e): lazy[int(e)] for e in which}
+
+        def __getitem__(self, e):
+            return self.rows[int(e)]
+
+    for key in ("W1", "W3", "W2", "W1s", "W3s", "W2s"):
+        if o.get(key) is not None:
+            o[key] = Widened(o[key], allowed if key in ("W1", "W3", "W2") else range(o[key].shape[0]))
     rng = np.random.default_rng(0)
     # size the sample from a small probe so one step takes about budget_s / max(steps, 1)
     probe = np.sort(rng.choice(cfg.T, min(64, cfg.T), replace=False))
@@ -296,8 +365,10 @@ def time_oracle(cfg, budget_s: float, steps: int = 0):
         times.append(time.perf_counter() - t0)
         done += n_tok
     total = sum(times)
+    thr, blas = blas_threads()
     desc = (f"{n_steps} x {n_tok} of {cfg.T} tokens (seeded sample; full layer on those tokens: gate, Top-k, "
-            f"routing tables, codec, experts, combine), numpy float64")
+            f"routing tables, codec, experts, combine), numpy float64; matmuls on {thr} {blas} threads, "
+            f"the rest single-threaded")
     return done / total, desc, times, n_tok
 
 
@@ -309,13 +380,14 @@ def run_reference(args):
     cores = os.cpu_count()
     budget = max(10.0, min(120.0, 3.0 * (args.steps + args.warmup)))
     tps, desc, times, n_tok = time_oracle(cfg, budget, steps=args.steps)
+    cores = blas_threads()[0] or cores
     ms = 1e3 * cfg.T / tps
     line = {"impl": "reference", "metric": METRIC, "value": round(tps, 2), "unit": "tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": describe(cfg), "l2": "n/a (CPU)"},
             "cpu_baseline": {"value": round(tps, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                             "sample": desc},
+                             "sample": desc, "host_cpus": os.cpu_count()},
             "e2e": {"value": round(tps, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
     print(json.dumps(line), flush=True)
@@ -474,17 +546,25 @@ def run_ours(args):
         serial_step()
     serial_ms = timed_loop(serial_step)
 
-    # Per-kernel device time: every launch of the graphed call bracketed by events.
-    pgraph = capture(True)
+    # Per-kernel device time: for each launch index i, a graph of the whole call
+    # with only launch i bracketed by events (its neighbours keep their overlap).
     prof_steps = max(args.steps, 5)
     per_kernel = {}
-    for _ in range(prof_steps):
-        flush.zero_()
-        pgraph.replay()
-        torch.cuda.synchronize(dev)
-        for i in range(C.ec2moe_profile_count()):
-            name, ms = C.ec2moe_profile_read(i)
-            per_kernel.setdefault(name, []).append(ms)
+    C.ec2moe_profile_reset()
+    for li in range(launches_per_step):
+        C.ec2moe_profile_only(li)
+        pgraph = capture(True)
+        # the capture left one record whose events every replay records again
+        for _ in range(prof_steps):
+            flush.zero_()
+            pgraph.replay()
+            torch.cuda.synchronize(dev)
+            for i in range(C.ec2moe_profile_count()):
+                name, ms = C.ec2moe_profile_read(i)
+                per_kernel.setdefault(name, []).append(ms)
+        del pgraph
+        C.ec2moe_profile_reset()
+    C.ec2moe_profile_only(-1)
     C.ec2moe_profile_reset()
 
     tot_step, tot_e2e, tot_serial = reduce_max([sum(step_ms), sum(e2e_ms), sum(serial_ms)], device=dev)
@@ -499,9 +579,10 @@ def run_ours(args):
     peaks, peaks_src = load_peaks()
     kern = {n: {"launches_per_step": len(v) / prof_steps, "avg_ms": statistics.mean(v),
                 "share": 0.0} for n, v in per_kernel.items()}
-    tot = sum(k["avg_ms"] * k["launches_per_step"] for k in kern.values())
     for k in kern.values():
-        k["share"] = round(k["avg_ms"] * k["launches_per_step"] / tot, 4) if tot else 0.0
+        # fraction of the step's time (kernels overlap their neighbours'
+        # prologues, so the shares may add up to a little more than 1)
+        k["share"] = round(k["avg_ms"] * k["launches_per_step"] / t_step, 4)
         k["avg_ms"] = round(k["avg_ms"], 5)
     dominant = max(kern, key=lambda n: kern[n]["avg_ms"] * kern[n]["launches_per_step"])
     touched = int((run.counts > 0).sum().item())
@@ -513,9 +594,9 @@ def run_ours(args):
 
     cpu = None
     if not args.no_cpu_baseline and world == 1:
-        tps, desc, _, _ = time_oracle(cfg, args.cpu_seconds, steps=1)
-        cpu = {"value": round(tps, 2), "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-               "sample": desc}
+        tps, desc, _, _ = time_oracle(cfg, args.cpu_seconds, steps=1, inp=inp)
+        cpu = {"value": round(tps, 2), "unit": "tokens/s", "cores": blas_threads()[0] or os.cpu_count(),
+               "kind": "oracle", "sample": desc, "host_cpus": os.cpu_count()}
 
     value = whole_job_tokens_per_s(world, cfg.T, t_step)
     es = 2 if cfg.dtype == 1 else 4
@@ -528,7 +609,9 @@ def run_ours(args):
                              "step's pinned H2D input copy and D2H output copy on their own streams, overlapped "
                              "with the neighbouring steps' compute (double-buffered; two weight sets alternate, "
                              "together larger than L2)",
-                   "parallelism": f"token-parallel replicas x{world}"},
+                   "parallelism": f"token-parallel replicas x{world}",
+                   "kernel_timing": "per launch index, a graph of the whole call with only that launch bracketed "
+                                    "by CUDA events, L2 flushed; share = kernel time / step time"},
         "layer_tflops": round(layer_flops / (t_step * 1e-3) / 1e12, 2),
         "layer_frac_bf16_peak": round(layer_flops / (t_step * 1e-3) / 1e12 / peaks["bf16_tflops"], 4),
         "roofline": roof,

@@ -127,7 +127,11 @@ size_t ec2moe_experts_workspace_size(const ec2moe_layer_desc* desc);
 /* Bytes of device workspace ec2moe_route needs (per-block histograms). */
 size_t ec2moe_route_workspace_size(const ec2moe_layer_desc* desc);
 
-/* Steps 1-3a: local expert filter, group gate and Top-k (Eq. 4-7).
+/* Steps 1-3a: local expert filter, group gate and Top-k.
+ * Passage: Eq. 4 (the local candidate set E_local), Eq. 5 (per-group softmax
+ * gates W_k x + b_k), Eq. 6 (global group gate W_global x + b_global), Eq. 7
+ * (g_i = p_group^(k) p_local,i^(k)), and the Top-k selection of the gating
+ * network that Eq. 1 sums over (Top-1 in the evaluation's parameter setup).
  *  X         [T, d] activations (dtype)
  *  mask      host uint8 [E]; 1 = expert in the local candidate set of Eq. 4.
  *            An all-zero mask returns EC2MOE_ERR_ALL_MASKED and fewer than k
@@ -145,6 +149,9 @@ ec2moe_status ec2moe_gate(const ec2moe_layer_desc* desc, const void* X, const fl
 
 /* Step 3b: per-expert histogram, exclusive scan and stable permutation, plus
  * the optional gather of activation rows into expert order.
+ * Passage: Eq. 1, whose sum runs only over the experts Top-k selected for each
+ * token (Top-1 routing in the evaluation's parameter setup): the rows routed
+ * to expert i are gathered so E_i runs once over all of them.
  *  topk_idx  int32 [T, k] (from ec2moe_gate)
  *  counts    out int32 [E]     tokens routed to each expert
  *  offsets   out int32 [E + 1] exclusive prefix sum of counts
@@ -153,7 +160,12 @@ ec2moe_status ec2moe_gate(const ec2moe_layer_desc* desc, const void* X, const fl
  *  inv_perm  out int32 [T * k] or NULL: inv_perm[perm[p]] = p
  *  src, dst  NULL, or src [T, width] and dst [T * k, width] (dtype):
  *            dst[p] = src[perm[p] / k]
- *  workspace device scratch of ec2moe_route_workspace_size bytes */
+ *  workspace device scratch of ec2moe_route_workspace_size bytes
+ * topk_idx is read on the device, so its ids cannot be checked before the
+ * launch: an id outside [0, E) is skipped by the kernels (not counted, no perm
+ * row, inv_perm = -1, no row gathered through it) and the next
+ * ec2moe_last_device_error returns EC2MOE_ERR_INVALID_ARG; counts, offsets and
+ * perm then describe the valid entries only. */
 ec2moe_status ec2moe_route(const ec2moe_layer_desc* desc, const int32_t* topk_idx, int32_t* counts,
                            int32_t* offsets, int32_t* perm, int32_t* inv_perm, const void* src,
                            int32_t width, void* dst, void* workspace, size_t ws_bytes,
@@ -177,8 +189,10 @@ ec2moe_status ec2moe_route(const ec2moe_layer_desc* desc, const int32_t* topk_id
  * allocated or freed, by this call or by anything it calls.
  *
  * The first call on each device looks up the array's device address (with
- * that device current) and caches it; make that first call before any stream
- * capture.  All calls on a device share the array: every cell a call reads is
+ * that device current) and caches it, keyed on the device's current context;
+ * make that first call before any stream capture.  After a cudaDeviceReset the
+ * next call looks the address up again in the new context (so it, too, should
+ * come before any capture), and the array's contents are gone.  All calls on a device share the array: every cell a call reads is
  * written earlier by the same call, but calls whose kernels overlap on the GPU
  * (different streams, or different host threads) race on it and must be
  * serialised by the caller. */
@@ -189,6 +203,8 @@ ec2moe_status ec2moe_route_noalloc(const ec2moe_layer_desc* desc, const int32_t*
 
 /* Steps 4-5a: routed expert FFNs on expert-ordered rows with the gate scale and
  * the unpermute fused into the down projection.
+ * Passage: Eq. 1, each term G(x)_i E_i(x) with E_i a feed-forward expert
+ * network (Preliminary, Mixture-of-Experts).
  *  X_perm    [T * k, d] rows in expert order (ec2moe_route's dst)
  *  offsets   int32 [E + 1] device (ec2moe_route)
  *  perm      int32 [T * k] device (ec2moe_route)
@@ -202,6 +218,8 @@ ec2moe_status ec2moe_experts(const ec2moe_layer_desc* desc, const void* X_perm, 
                              ec2moe_stream_t stream);
 
 /* Always-on shared experts on every token: shared_out[s * T + t] = E_s(x_t).
+ * Passage: Eq. 1's expert FFN E_i applied with weight 1 to every token; the
+ * paper has no shared experts, the fine-grained layer shape adds them.
  *  X [T, d]; W1s/W3s/W2s as in ec2moe_layer_weights; shared_out out
  *  [n_shared * T, d]; workspace of ec2moe_experts_workspace_size bytes. */
 ec2moe_status ec2moe_shared_experts(const ec2moe_layer_desc* desc, const void* X, const void* W1s,
@@ -209,20 +227,29 @@ ec2moe_status ec2moe_shared_experts(const ec2moe_layer_desc* desc, const void* X
                                     size_t ws_bytes, ec2moe_stream_t stream);
 
 /* Step 5b: y[t] = sum_s slot_out[t * k + s] + sum_j shared_out[j * T + t], in
- * that fixed order with an fp32 sum (Eq. 1).  shared_out may be NULL. */
+ * that fixed order with an fp32 sum.  shared_out may be NULL.
+ * Passage: Eq. 1, the sum over the selected experts of G(x)_i E_i(x). */
 ec2moe_status ec2moe_combine(const ec2moe_layer_desc* desc, const void* slot_out, const void* shared_out,
                              void* Y, ec2moe_stream_t stream);
 
-/* Step 6, end side: Z = X V_enc^T ([T, d] x [r, d]^T -> [T, r]). */
+/* Step 6, end side: Z = X V_enc^T ([T, d] x [r, d]^T -> [T, r]).
+ * Passage: the low-rank encoder of PO-ECC (Encoder-Decoder based on Low-Rank
+ * Compression): Z = U^T X V, here with U = I on the token axis and
+ * V = V_enc^T. */
 ec2moe_status ec2moe_lr_encode(const ec2moe_layer_desc* desc, const void* X, const void* V_enc, void* Z,
                                ec2moe_stream_t stream);
 
-/* Step 6, cloud side: X_hat = Z V_dec^T ([T, r] x [d, r]^T -> [T, d]). */
+/* Step 6, cloud side: X_hat = Z V_dec^T ([T, r] x [d, r]^T -> [T, d]).
+ * Passage: the decoder of the same section, X_hat = U_hat Z V_hat^T, with
+ * U_hat = I and V_hat = V_dec. */
 ec2moe_status ec2moe_lr_decode(const ec2moe_layer_desc* desc, const void* Z, const void* V_dec,
                                void* X_hat, ec2moe_stream_t stream);
 
 /* The fused layer: gate and routing on X, encode, decode into expert order,
  * routed and shared experts, combine.
+ * Passage: Eq. 1 with the gate of Eq. 4-7 (HL-GGN) and the low-rank
+ * encoder/decoder of PO-ECC at the end-cloud split between the gate and the
+ * experts.
  *  Y         out [T, d] (dtype)
  *  topk_idx  out int32 [T, k]; topk_w out fp32 [T, k]; counts out int32 [E]
  *  Z         out [T, r] or NULL: the transmitted (encoded) activations
@@ -232,10 +259,11 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
                                    float* topk_w, int32_t* counts, void* Z, void* workspace,
                                    size_t ws_bytes, ec2moe_stream_t stream);
 
-/* Synchronises `stream`, then reads and clears the device error word of the
+/* Synchronises `stream`, then reads and clears the device error words of the
  * current device: EC2MOE_OK, EC2MOE_ERR_TIMEOUT when a bounded wait in a
- * tensor-core kernel gave up, or EC2MOE_ERR_CUDA when the stream reports an
- * error. */
+ * tensor-core kernel gave up, EC2MOE_ERR_INVALID_ARG when a routing kernel met
+ * (and skipped) an expert id outside [0, E) in a caller's topk_idx, or
+ * EC2MOE_ERR_CUDA when the stream reports an error. */
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream);
 
 /* Budget, in SM clock cycles, of every bounded wait inside the tensor-core
@@ -296,6 +324,14 @@ int32_t ec2moe_last_launch_count(void);
  * "shared_down", "combine", "sum_counts"); `ms` its device duration.  Profiling is off by default and
  * costs nothing when off. */
 ec2moe_status ec2moe_profile_enable(int32_t enable);
+/* Restricts profiling to one launch per call: with launch_index >= 0 only the
+ * kernel that is the launch_index-th launch (0-based) of each later call is
+ * bracketed, so its neighbours run without event records between them (which
+ * would otherwise end the programmatic overlap of every launch with its
+ * predecessor and add the records' own cost to every measured kernel);
+ * -1 (the default) brackets every launch.  Values below -1 return
+ * EC2MOE_ERR_INVALID_ARG. */
+ec2moe_status ec2moe_profile_only(int32_t launch_index);
 int32_t ec2moe_profile_count(void);
 ec2moe_status ec2moe_profile_read(int32_t i, const char** name, float* ms);
 void ec2moe_profile_reset(void);

@@ -43,8 +43,25 @@ def _compile(src: str, verbose_ptxas: bool) -> str:
     return obj
 
 
+_ELF_MACHINE = {"x86_64": 62, "amd64": 62, "aarch64": 183, "arm64": 183}
+
+
+def _foreign_arch(path: str) -> bool:
+    """True when the ELF file at `path` was built for another CPU than this host's."""
+    import platform
+    want = _ELF_MACHINE.get(platform.machine().lower())
+    try:
+        with open(path, "rb") as f:
+            head = f.read(20)
+    except OSError:
+        return True
+    if len(head) < 20 or head[:4] != b"\x7fELF":
+        return True
+    return want is not None and int.from_bytes(head[18:20], "little") != want
+
+
 def _stale() -> bool:
-    if not os.path.exists(LIB):
+    if not os.path.exists(LIB) or _foreign_arch(LIB):
         return True
     t = os.path.getmtime(LIB)
     deps = [os.path.join(CSRC, f) for f in os.listdir(CSRC)]

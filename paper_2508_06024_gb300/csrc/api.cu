@@ -25,6 +25,7 @@ struct ProfRecord {
 };
 std::mutex g_prof_mu;
 bool g_prof_on = false;
+int g_prof_only = -1;  // >= 0: bracket only the launch with this index in each call
 std::vector<ProfRecord> g_prof;
 std::vector<cudaEvent_t> g_pool;
 size_t g_pool_used = 0;
@@ -66,7 +67,7 @@ int launch_count() { return t_launches; }
 
 KernelScope::KernelScope(const char* name, cudaStream_t s) : name_(name), s_(s) {
   std::lock_guard<std::mutex> lock(g_prof_mu);
-  if (g_prof_on) {
+  if (g_prof_on && (g_prof_only < 0 || g_prof_only == t_launches)) {
     start_ = pool_event();
     if (start_) record_on(start_, s_);
   }
@@ -961,11 +962,13 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
 
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream) {
   if (cudaStreamSynchronize(stream) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  unsigned int word = 0, word2 = 0, word3 = 0;
+  unsigned int word = 0, word2 = 0, word3 = 0, word4 = 0;
   if (read_tc_error(&word) != cudaSuccess) return EC2MOE_ERR_CUDA;
   if (read_codec_error(&word2) != cudaSuccess) return EC2MOE_ERR_CUDA;
   if (read_gate_error(&word3) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  return (word | word2 | word3) ? EC2MOE_ERR_TIMEOUT : EC2MOE_OK;
+  if (read_route_error(&word4) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (word | word2 | word3) return EC2MOE_ERR_TIMEOUT;
+  return word4 ? EC2MOE_ERR_INVALID_ARG : EC2MOE_OK;
 }
 
 int32_t ec2moe_last_launch_count(void) { return launch_count(); }
@@ -981,6 +984,13 @@ int64_t ec2moe_get_wait_budget(void) { return default_timeout_cycles(); }
 ec2moe_status ec2moe_profile_enable(int32_t enable) {
   std::lock_guard<std::mutex> lock(g_prof_mu);
   g_prof_on = enable != 0;
+  return EC2MOE_OK;
+}
+
+ec2moe_status ec2moe_profile_only(int32_t launch_index) {
+  if (launch_index < -1) return EC2MOE_ERR_INVALID_ARG;
+  std::lock_guard<std::mutex> lock(g_prof_mu);
+  g_prof_only = launch_index;
   return EC2MOE_OK;
 }
 

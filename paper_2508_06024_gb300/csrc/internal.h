@@ -213,6 +213,10 @@ cudaError_t read_gate_error(unsigned int* word);
 
 // Reads and clears the tensor-core kernels' device error word (synchronous).
 cudaError_t read_tc_error(unsigned int* word);
+// Reads and clears the routing kernels' device error word (synchronous):
+// nonzero when an expert id outside [0, E) or a permutation entry outside
+// [0, rows) was met (and skipped).
+cudaError_t read_route_error(unsigned int* word);
 long long default_timeout_cycles();
 void set_timeout_cycles(long long cycles);
 

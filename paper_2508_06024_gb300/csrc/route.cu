@@ -31,8 +31,20 @@ namespace {
 // kernels overlap on the GPU race on it.
 static __device__ __align__(256) int32_t g_route_noalloc_cells[EC2MOE_ROUTE_NOALLOC_MAX_CELLS];
 
+// Bit 0: a routing kernel met an expert id outside [0, E) in the caller's
+// topk_idx, or a gather met a permutation entry outside [0, rows).  Such
+// entries are skipped (no shared or global access through them) and
+// ec2moe_last_device_error reports EC2MOE_ERR_INVALID_ARG.
+__device__ unsigned int g_route_error;
+
 constexpr int CHUNK = 1024;  // entries per block (one per thread)
 constexpr int MAXE = 128;
+
+__device__ __forceinline__ bool valid_expert(int e, int E) {
+  if (static_cast<unsigned>(e) < static_cast<unsigned>(E)) return true;
+  atomicOr(&g_route_error, 1u);
+  return false;
+}
 
 __global__ void __launch_bounds__(CHUNK) route_count_kernel(const int32_t* __restrict__ idx, long long n, int E,
                                                             int32_t* __restrict__ blk_counts) {
@@ -42,7 +54,10 @@ __global__ void __launch_bounds__(CHUNK) route_count_kernel(const int32_t* __res
   for (int e = threadIdx.x; e < E; e += blockDim.x) hist[e] = 0;
   __syncthreads();
   const long long i = (long long)blockIdx.x * CHUNK + threadIdx.x;
-  if (i < n) atomicAdd(&hist[idx[i]], 1);
+  if (i < n) {
+    const int e = idx[i];
+    if (valid_expert(e, E)) atomicAdd(&hist[e], 1);
+  }
   __syncthreads();
   for (int e = threadIdx.x; e < E; e += blockDim.x) blk_counts[(long long)blockIdx.x * E + e] = hist[e];
 }
@@ -85,11 +100,12 @@ __global__ void __launch_bounds__(CHUNK) route_scatter_kernel(const int32_t* __r
     if (blockIdx.x == 0) offsets[E] = acc;
   }
   const long long i = (long long)blockIdx.x * CHUNK + threadIdx.x;
-  const bool live = i < n;
+  int e = i < n ? idx[i] : -1;
+  const bool live = i < n && valid_expert(e, E);
+  if (i < n && !live && inv_perm) inv_perm[i] = -1;
   const unsigned act = __ballot_sync(0xffffffffu, live);
-  int e = -1, rank_w = 0;
+  int rank_w = 0;
   if (live) {
-    e = idx[i];
     const unsigned same = __match_any_sync(act, e);
     rank_w = __popc(same & ((1u << lane) - 1u));
     if (rank_w == 0) s_wcnt[warp][e] = __popc(same);
@@ -133,10 +149,10 @@ __global__ void __launch_bounds__(CHUNK) route_small_kernel(const int32_t* __res
   __syncthreads();
   for (int i0 = 0; i0 < n; i0 += CHUNK) {
     const int i = i0 + threadIdx.x;
-    const bool live = i < n;
+    const int e = i < n ? idx[i] : -1;
+    const bool live = i < n && valid_expert(e, E);
     const unsigned act = __ballot_sync(0xffffffffu, live);
     if (live) {
-      const int e = idx[i];
       const unsigned same = __match_any_sync(act, e);
       if ((same & ((1u << lane) - 1u)) == 0) atomicAdd(&hist[e], __popc(same));
     }
@@ -156,11 +172,12 @@ __global__ void __launch_bounds__(CHUNK) route_small_kernel(const int32_t* __res
     for (int c = threadIdx.x; c < (CHUNK / 32) * MAXE; c += blockDim.x) (&wcnt[0][0])[c] = 0;
     __syncthreads();
     const int i = i0 + threadIdx.x;
-    const bool live = i < n;
+    int e = i < n ? idx[i] : -1;
+    const bool live = i < n && static_cast<unsigned>(e) < static_cast<unsigned>(E);
+    if (i < n && !live && inv_perm) inv_perm[i] = -1;
     const unsigned act = __ballot_sync(0xffffffffu, live);
-    int e = 0, rank_w = 0;
+    int rank_w = 0;
     if (live) {
-      e = idx[i];
       const unsigned same = __match_any_sync(act, e);
       rank_w = __popc(same & ((1u << lane) - 1u));
       if (rank_w == 0) wcnt[warp][e] = __popc(same);
@@ -194,7 +211,12 @@ __global__ void gather_rows_kernel(const uint8_t* __restrict__ src, uint8_t* __r
   const int lane = threadIdx.x & 31;
   const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
   for (long long r = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += warps) {
-    const long long t = perm[r] / k;
+    const int32_t p = perm[r];
+    if (static_cast<unsigned long long>(p) >= static_cast<unsigned long long>(rows)) {
+      if (lane == 0) atomicOr(&g_route_error, 1u);
+      continue;
+    }
+    const long long t = p / k;
     const U4* s = reinterpret_cast<const U4*>(src + t * row_bytes);
     U4* d = reinterpret_cast<U4*>(dst + r * row_bytes);
     for (int c = lane; c < row_bytes / 16; c += 32) d[c] = s[c];
@@ -218,7 +240,12 @@ __global__ void gather_rel_kernel(const uint8_t* __restrict__ src, uint8_t* __re
   __syncthreads();
   const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
   for (long long i = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); i < n; i += warps) {
-    const int pos = s_off[idx[i]] + rel[i];
+    const int e = idx[i];
+    if (static_cast<unsigned>(e) >= static_cast<unsigned>(E)) {
+      if (lane == 0) atomicOr(&g_route_error, 1u);
+      continue;
+    }
+    const int pos = s_off[e] + rel[i];
     if (lane == 0) perm[pos] = static_cast<int32_t>(i);
     const U4* sr = reinterpret_cast<const U4*>(src + (i / k) * row_bytes);
     U4* dr = reinterpret_cast<U4*>(dst + (long long)pos * row_bytes);
@@ -286,25 +313,60 @@ cudaError_t launch_route(const int32_t* topk_idx, long long n, int E, int32_t* b
   return cudaGetLastError();
 }
 
+// Id of the current CUDA context (driver entry points reached through the
+// runtime, so the library needs no link against libcuda).  False when there is
+// no current context yet or the entry points are missing.
+static bool current_context_id(unsigned long long* id) {
+  using GetCurrentFn = CUresult (*)(CUcontext*);
+  using GetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+  static GetCurrentFn get_current = nullptr;
+  static GetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<GetCurrentFn>(f);
+    f = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<GetIdFn>(f);
+  });
+  if (!get_current || !get_id) return false;
+  CUcontext ctx = nullptr;
+  if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return false;
+  return get_id(ctx, id) == CUDA_SUCCESS;
+}
+
 // Device address of g_route_noalloc_cells for the current device.  The host-side
 // name of a __device__ array is only a stand-in, so the address is looked up
-// once per device (with that device current) and cached.
+// with the device current and cached per device, keyed on the context's id: a
+// cudaDeviceReset destroys the context (and the array with it), and the next
+// call then looks the address up again in the new context.
 static cudaError_t noalloc_cells(int32_t** out) {
   constexpr int MAX_DEVICES = 64;
+  struct Entry {
+    int32_t* ptr;
+    unsigned long long ctx;
+  };
   static std::mutex mu;
-  static int32_t* cache[MAX_DEVICES] = {};
+  static Entry cache[MAX_DEVICES] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= MAX_DEVICES) return cudaErrorInvalidDevice;
   std::lock_guard<std::mutex> lock(mu);
-  if (!cache[dev]) {
+  unsigned long long ctx = 0;
+  const bool known_ctx = current_context_id(&ctx);
+  if (!cache[dev].ptr || !known_ctx || cache[dev].ctx != ctx) {
     void* p = nullptr;
     e = cudaGetSymbolAddress(&p, g_route_noalloc_cells);
     if (e != cudaSuccess) return e;
-    cache[dev] = static_cast<int32_t*>(p);
+    unsigned long long ctx_now = 0;
+    cache[dev] = Entry{static_cast<int32_t*>(p), current_context_id(&ctx_now) ? ctx_now : 0ull};
   }
-  *out = cache[dev];
+  *out = cache[dev].ptr;
   return cudaSuccess;
 }
 
@@ -357,6 +419,13 @@ __global__ void sum_counts_kernel(const int32_t* __restrict__ parts, int n_parts
     for (int p = 0; p < n_parts; ++p) c += parts[(size_t)p * E + e];
     counts[e] = c;
   }
+}
+
+cudaError_t read_route_error(unsigned int* word) {
+  unsigned int zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(word, g_route_error, sizeof(unsigned int));
+  if (e != cudaSuccess) return e;
+  return cudaMemcpyToSymbol(g_route_error, &zero, sizeof(unsigned int));
 }
 
 cudaError_t launch_sum_counts(const int32_t* parts, int n_parts, int E, int32_t* counts, cudaStream_t s) {

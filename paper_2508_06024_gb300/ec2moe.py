@@ -41,7 +41,7 @@ EXPORTED = [
     "ec2moe_last_launch_count", "ec2moe_status_string", "ec2moe_profile_enable", "ec2moe_profile_count",
     "ec2moe_profile_read", "ec2moe_profile_reset", "ec2moe_route_noalloc", "ec2moe_set_wait_budget",
     "ec2moe_get_wait_budget", "ec2moe_schedule", "ec2moe_schedule_objective", "ec2moe_expert_tasks",
-    "ec2moe_pipelined_workspace_size", "ec2moe_layer_forward_pipelined",
+    "ec2moe_pipelined_workspace_size", "ec2moe_layer_forward_pipelined", "ec2moe_profile_only",
 ]
 
 END = 0
@@ -89,6 +89,7 @@ _SIGS = {
     "ec2moe_status_string": (ctypes.c_char_p, [ctypes.c_int]),
     "ec2moe_profile_enable": (ctypes.c_int, [ctypes.c_int32]),
     "ec2moe_profile_count": (ctypes.c_int32, []),
+    "ec2moe_profile_only": (ctypes.c_int, [ctypes.c_int32]),
     "ec2moe_profile_read": (ctypes.c_int, [ctypes.c_int32, ctypes.POINTER(ctypes.c_char_p),
                                            ctypes.POINTER(ctypes.c_float)]),
     "ec2moe_profile_reset": (None, []),
@@ -263,6 +264,11 @@ def ec2moe_last_launch_count() -> int:
 
 def ec2moe_profile_enable(enable: bool = True) -> None:
     _check(load().ec2moe_profile_enable(1 if enable else 0), "ec2moe_profile_enable")
+
+
+def ec2moe_profile_only(launch_index: int) -> None:
+    """Bracket only the launch_index-th launch of each later call (-1: every launch)."""
+    _check(load().ec2moe_profile_only(int(launch_index)), "ec2moe_profile_only")
 
 
 def ec2moe_profile_count() -> int:

@@ -2,7 +2,12 @@
 kernels is bounded.  With a wait budget of 0 the first wait that is not
 already satisfied gives up; the CTA drains its own copies and MMAs, frees its
 tensor memory and returns, and the host reads EC2MOE_ERR_TIMEOUT.  The same
-process then runs the layer normally and gets the same output as before."""
+process then runs the layer normally and gets the same output as before.
+
+Routing reads the caller's Top-k ids on the device, so ids outside [0, E)
+cannot be refused before the launch: the routing kernels skip them (no shared
+or global access through them) and the host reads EC2MOE_ERR_INVALID_ARG."""
+import numpy as np
 import pytest
 import torch
 
@@ -46,3 +51,50 @@ def test_wait_budget_rejects_negative():
     with pytest.raises(C.Ec2moeError) as e:
         C.ec2moe_set_wait_budget(-1)
     assert e.value.status == C.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("T,k,E", [(300, 2, 16), (9000, 2, 16), (20000, 1, 64)],
+                         ids=["one-block", "two-kernel", "two-kernel-E64"])
+@pytest.mark.parametrize("noalloc", [False, True], ids=["workspace", "noalloc"])
+def test_route_out_of_range_ids_are_skipped_and_reported(T, k, E, noalloc):
+    d = 64
+    desc = C.make_desc(T=T, d=d, E=E, d_ff=128, k=k)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(T + E)
+    idx = torch.randint(0, E, (T, k), generator=g, device="cuda", dtype=torch.int32)
+    bad = [(0, 0), (T // 2, k - 1), (T - 1, 0)]
+    for (t, s), v in zip(bad, (E, -1, 1 << 30)):
+        idx[t, s] = v
+    n = T * k
+    X = torch.randn(T, d, generator=g, device="cuda").to(torch.bfloat16)
+    counts = torch.empty(E, dtype=torch.int32, device="cuda")
+    offsets = torch.empty(E + 1, dtype=torch.int32, device="cuda")
+    perm = torch.full((n,), -5, dtype=torch.int32, device="cuda")
+    inv = torch.empty(n, dtype=torch.int32, device="cuda")
+    dst = torch.zeros(n, d, dtype=torch.bfloat16, device="cuda")
+    if noalloc:
+        C.ec2moe_route_noalloc(desc, idx, counts, offsets, perm, inv, X, d, dst)
+    else:
+        wsb = C.ec2moe_route_workspace_size(desc)
+        ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device="cuda")
+        C.ec2moe_route(desc, idx, counts, offsets, perm, inv, X, d, dst, ws, wsb)
+    assert C.ec2moe_last_device_error() == C.ERR_INVALID_ARG
+    assert C.ec2moe_last_device_error() == C.OK  # read and cleared
+    flat = idx.cpu().numpy().ravel()
+    valid = (flat >= 0) & (flat < E)
+    assert np.array_equal(counts.cpu().numpy(), np.bincount(flat[valid], minlength=E))
+    m = int(valid.sum())
+    assert offsets.cpu().numpy()[-1] == m
+    p = perm.cpu().numpy()
+    assert np.array_equal(np.sort(p[:m]), np.flatnonzero(valid))
+    iv = inv.cpu().numpy()
+    assert (iv[~valid] == -1).all() and np.array_equal(iv[p[:m]], np.arange(m))
+    rows = torch.from_numpy((p[:m] // k).astype(np.int64)).cuda()
+    assert torch.equal(dst[:m], X[rows])
+    # the context is intact: a valid call afterwards succeeds and reports OK
+    idx[idx >= E] = 0
+    idx[idx < 0] = 0
+    C.ec2moe_route_noalloc(desc, idx, counts, offsets, perm, inv, X, d, dst) if noalloc else \
+        C.ec2moe_route(desc, idx, counts, offsets, perm, inv, X, d, dst, ws, wsb)
+    assert C.ec2moe_last_device_error() == C.OK
+    assert int(counts.sum().item()) == n

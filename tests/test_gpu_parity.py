@@ -75,7 +75,11 @@ def test_gate_topk(cfg):
     ref = _gate_ref(cfg, inp)
     gi, gw = idx.cpu().numpy(), w.cpu().numpy()
     n_cmp, n_excl = routing_check(gi, ref)
-    assert n_excl <= max(2, cfg.T // 1000), n_excl
+    # A token is excluded when its k-th and (k+1)-th choices are within 1e-6
+    # in log g.  Those gaps have a density of order one near zero, so about
+    # T * 1e-6 tokens (well below one at these sizes) are expected; the bound
+    # leaves room for a few without hiding a systematic difference.
+    assert n_excl <= max(2, cfg.T // 8192), n_excl
     weights_check(gi, gw, ref, ref["gap_boundary"] >= TIE_GAP)
     # masked experts never selected; counts over the kept tokens agree exactly
     mask = inp["mask"].cpu().numpy()
@@ -258,6 +262,43 @@ def test_layer_forward(cfg, sample):
     if cfg.r > 0:
         Z = _np(run.Z)[sel]
         output_check(Z, ref["Z"], cfg.dtype == S.BF16)
+
+
+@pytest.mark.parametrize("cfg", [S.preset("mixtral_bf16"), S.preset("finegrained_bf16"),
+                                 S.preset("switch_bf16", T=65536, seed=48)], ids=lambda c: c.name + f"-T{c.T}")
+def test_layer_sample_covers_a_partial_tail_tile(cfg):
+    """At full size the output is checked on a sample of rows; this sample
+    always holds every row of one expert group smaller than a 128-row m-tile,
+    so a group whose only tile is partial (its tail) is checked whole.  The
+    least-loaded allowed expert's local bias is lowered until it receives
+    between 1 and 127 rows."""
+    inp = S.make_inputs(cfg, device="cuda")
+    run = LayerRun(cfg, inp)
+    run.forward()
+    torch.cuda.synchronize()
+    allowed = np.flatnonzero(inp["mask"].cpu().numpy())
+    e = int(allowed[np.argmin(run.counts.cpu().numpy()[allowed])])
+    base = float(inp["b_local"][e])
+    for shift in (0.0, 1.0, 2.0, 3.0, 4.0, 5.0, 6.0, 8.0, 10.0, 13.0):
+        inp["b_local"][e] = base - shift
+        run.forward()
+        torch.cuda.synchronize()
+        c = int(run.counts[e])
+        if 1 <= c <= 127:
+            break
+    assert 1 <= c <= 127, c
+    assert C.ec2moe_last_device_error() == C.OK
+    gi = run.topk_idx.cpu().numpy()
+    group_rows = np.flatnonzero((gi == e).any(axis=1))
+    rng = np.random.default_rng(cfg.seed + 7)
+    rows = np.union1d(group_rows, rng.choice(cfg.T, 128, replace=False))
+    ref = orc.layer_forward(oracle_inputs(inp, lazy_experts=True), cfg.n_groups, cfg.k, cfg.act,
+                            bool(cfg.renorm_topk), rows=rows)
+    routing_check(gi, ref)
+    assert np.array_equal(run.counts.cpu().numpy(), np.bincount(gi.ravel(), minlength=cfg.E))
+    keep = ref["gap_boundary"][rows] >= TIE_GAP
+    assert keep[np.isin(rows, group_rows)].sum() >= len(group_rows) - 2
+    output_check(_np(run.Y)[rows][keep], ref["y"][keep], True)
 
 
 def test_layer_is_deterministic():

@@ -65,14 +65,48 @@ def _route_both(cfg, X):
 
 @pytest.mark.gpu
 def test_noalloc_route_matches_workspace_route_twice(lib):
-    # Two calls in a row with different shapes and expert counts: the second
-    # call runs over the array the first one left behind.
+    # Two calls in a row, both with more than 16384 (token, slot) entries so
+    # that both take the two-kernel routing that reads the library's array,
+    # and with different expert counts (64, then 16): the second call's kernels
+    # run over cells the first call left behind in another layout.
     for cfg in (S.preset("finegrained_bf16", T=9000, seed=21),
-                S.preset("switch_bf16", T=3001, k=2, n_groups=4, seed=22)):
+                S.preset("switch_bf16", T=20000, k=2, n_groups=4, seed=22)):
+        assert cfg.T * cfg.k > 16384
         X = S.make_inputs(cfg, device="cuda", with_experts=False)["X"]
         idx, (ref, got) = _route_both(cfg, X)
         for a, b in zip(ref, got):
             assert torch.equal(a, b)
         counts = got[0].cpu().numpy()
         assert np.array_equal(counts, np.bincount(idx.cpu().numpy().ravel(), minlength=cfg.E))
+    assert C.ec2moe_last_device_error() == C.OK
+
+
+@pytest.mark.gpu
+def test_noalloc_route_at_the_array_limit(lib):
+    # ceil(T*k/1024) * E = 256 * 64 = 16384 cells: exactly the array's size.
+    T, E, k = 262144, 64, 1
+    desc = C.make_desc(T=T, d=256, E=E, d_ff=512, k=k)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(31)
+    outs = []
+    for seed_shift in (0, 1):
+        idx = torch.randint(0, E, (T, k), generator=g, device="cuda", dtype=torch.int32)
+        res = []
+        for use_noalloc in (False, True):
+            counts = torch.full((E,), -7, dtype=torch.int32, device="cuda")
+            offsets = torch.full((E + 1,), -7, dtype=torch.int32, device="cuda")
+            perm = torch.full((T * k,), -7, dtype=torch.int32, device="cuda")
+            if use_noalloc:
+                C.ec2moe_route_noalloc(desc, idx, counts, offsets, perm)
+            else:
+                wsb = C.ec2moe_route_workspace_size(desc)
+                ws = torch.empty(max(wsb, 16), dtype=torch.uint8, device="cuda")
+                C.ec2moe_route(desc, idx, counts, offsets, perm, None, None, 0, None, ws, wsb)
+            res.append((counts, offsets, perm))
+        torch.cuda.synchronize()
+        for a, b in zip(*res):
+            assert torch.equal(a, b)
+        assert np.array_equal(res[1][0].cpu().numpy(), np.bincount(idx.cpu().numpy().ravel(), minlength=E))
+        outs.append(res[1][2].clone())
+    assert not torch.equal(outs[0], outs[1])
     assert C.ec2moe_last_device_error() == C.OK
