@@ -62,3 +62,36 @@ class LayerRun:
                                self.topk_idx, self.topk_w, self.counts, self.Z, self.workspace, self.ws_bytes,
                                stream)
         return self.Y
+
+
+def main(argv=None) -> int:
+    """Runs `--calls` eager layer calls of a preset shape (for profilers such as
+    ncu, which want a short program with a known launch sequence)."""
+    import argparse
+
+    from . import build as B
+    from . import synth as S
+
+    ap = argparse.ArgumentParser(description="run a preset MoE layer shape through the C ABI")
+    ap.add_argument("--workload", default="mixtral_bf16")
+    ap.add_argument("--calls", type=int, default=2)
+    for key in ("T", "E", "n_allowed", "k", "r", "d_ff", "n_groups", "seed"):
+        ap.add_argument(f"--{key}", type=int, default=None)
+    args = ap.parse_args(argv)
+    over = {k: getattr(args, k) for k in ("T", "E", "n_allowed", "k", "r", "d_ff", "n_groups", "seed")
+            if getattr(args, k) is not None}
+    cfg = S.preset(args.workload, **over)
+    B.build()
+    C.load()
+    run = LayerRun(cfg, S.make_inputs(cfg, device="cuda"), device="cuda")
+    for _ in range(args.calls):
+        run.forward()
+    status = C.ec2moe_last_device_error()
+    torch.cuda.synchronize()
+    print(f"{cfg}: {args.calls} calls, {C.ec2moe_last_launch_count()} launches per call, "
+          f"status {C.status_string(status)}")
+    return 0 if status == C.OK else 1
+
+
+if __name__ == "__main__":
+    raise SystemExit(main())
