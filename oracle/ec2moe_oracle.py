@@ -18,6 +18,9 @@ Steps and the passages they follow:
   stacked into one [E, d] matrix) and Eq. 6 (W_global x + b_global).
 * ``group_gate``        - Eq. 5 (per-group softmax), Eq. 6 (group softmax) and
   Eq. 7 (g_i = p_group^(k) * p_local,i^(k)), restricted to allowed experts.
+* ``group_gate_pruned`` - the hierarchical use of Eq. 5-7 with top-group
+  pruning: Eq. 6 first, then Eq. 5 only inside the top groups, then Eq. 7
+  (the "lightweight" evaluation the group gate section motivates).
 * ``topk_route``        - Top-k selection (Top-1 in the evaluation setup),
   ties to the lower expert index.
 * ``route_tables``      - per-expert histogram, exclusive scan and the stable
@@ -145,6 +148,66 @@ def group_gate(l: np.ndarray, m: Optional[np.ndarray], allowed: np.ndarray, n_gr
     return g, log_g
 
 
+def pruned_candidate_floor(allowed: np.ndarray, n_groups: int, top_groups: int) -> int:
+    """Fewest allowed experts that any choice of ``top_groups`` live groups holds
+    (the sum of the smallest per-group allowed counts); Top-k needs k of them."""
+    E = allowed.shape[0]
+    b = group_bounds(E, n_groups)
+    sizes = sorted(int(allowed[b[j]:b[j + 1]].sum()) for j in range(n_groups) if allowed[b[j]:b[j + 1]].any())
+    return int(sum(sizes[:top_groups]))
+
+
+def group_gate_pruned(l: np.ndarray, m: np.ndarray, allowed: np.ndarray, n_groups: int, top_groups: int):
+    """Eq. 5-7 evaluated hierarchically with top-group pruning.
+
+    Per token, in the paper's order:
+      1. Eq. 6: the group probabilities p_group = softmax of m over the live
+         groups (those with an allowed member).
+      2. Keep the ``top_groups`` live groups with the largest p_group (ties to
+         the lower group index); the others are pruned for this token.
+      3. Eq. 5 only inside the kept groups: p_local = softmax of l over the
+         allowed members of each kept group.
+      4. Eq. 7: g_i = p_group'^(k) * p_local,i, where p_group' is p_group
+         renormalised over the kept groups, so that the gate still sums to 1
+         over its candidates as Eq. 1 requires.  Experts of pruned groups (and
+         masked experts) get g = 0 and log g = -inf.
+    ``top_groups`` >= the number of live groups keeps every live group, which
+    is ``group_gate`` itself.  Returns (g [T, E], log_g [T, E], group_gap [T]):
+    group_gap is the margin in m between the last kept group and the best
+    pruned one (+inf when nothing is pruned), used to exclude near-ties of the
+    group decision from exact checks.
+    """
+    T, E = l.shape
+    bounds = group_bounds(E, n_groups)
+    live = [j for j in range(n_groups) if allowed[bounds[j]:bounds[j + 1]].any()]
+    g = np.zeros((T, E))
+    log_g = np.full((T, E), -np.inf)
+    group_gap = np.full(T, np.inf)
+    for t in range(T):
+        # step 1: Eq. 6 over the live groups
+        p_group = np.exp(m[t, live] - m[t, live].max())
+        p_group /= p_group.sum()
+        # step 2: the top groups by p_group, ties to the lower group index
+        ranked = sorted(range(len(live)), key=lambda q: (-p_group[q], live[q]))
+        kept = sorted(live[q] for q in ranked[:top_groups])
+        if top_groups < len(live):
+            group_gap[t] = m[t, live[ranked[top_groups - 1]]] - m[t, live[ranked[top_groups]]]
+        # step 4's renormalised group probabilities over the kept groups
+        mk = m[t, kept]
+        lse_kept = mk.max() + np.log(np.exp(mk - mk.max()).sum())
+        for j in kept:
+            lo, hi = bounds[j], bounds[j + 1]
+            members = [i for i in range(lo, hi) if allowed[i]]
+            # step 3: Eq. 5 inside the kept group
+            z = l[t, members]
+            lse_j = z.max() + np.log(np.exp(z - z.max()).sum())
+            log_pg = m[t, j] - lse_kept
+            for i, zi in zip(members, z):
+                log_g[t, i] = log_pg + (zi - lse_j)
+                g[t, i] = np.exp(log_g[t, i])
+    return g, log_g, group_gap
+
+
 def topk_route(g: np.ndarray, allowed: np.ndarray, k: int):
     """Top-k experts per token by g, ties to the lower expert index.
 
@@ -244,21 +307,37 @@ def expert_ffn(x: np.ndarray, W1: np.ndarray, W2: np.ndarray, W3: Optional[np.nd
     return h @ np.asarray(W2, dtype=np.float64).T
 
 
-def gate_and_route(X, W_local, b_local, W_global, b_global, mask, n_groups: int, k: int, renorm: bool = False):
-    """Steps 1-3 for all tokens: mask, group gate, top-k, tables and margins."""
+def gate_and_route(X, W_local, b_local, W_global, b_global, mask, n_groups: int, k: int, renorm: bool = False,
+                   top_groups: int = 0):
+    """Steps 1-3 for all tokens: mask, group gate, top-k, tables and margins.
+
+    ``top_groups`` > 0 (with n_groups > 1) applies top-group pruning
+    (``group_gate_pruned``); k must then not exceed the allowed experts the
+    fewest-member choice of top_groups live groups holds.  With pruning the
+    boundary margin also covers the group decision (the smaller of the two)."""
     allowed = allowed_experts(mask, k)
     l, m = gate_logits(X, W_local, b_local, W_global, b_global)
-    g, log_g = group_gate(l, m, allowed, n_groups)
-    idx = topk_route(g, allowed, k)
+    pruned = top_groups > 0 and n_groups > 1
+    if pruned:
+        if pruned_candidate_floor(allowed, n_groups, top_groups) < k:
+            raise ValueError("fewer allowed experts in the kept groups than k")
+        g, log_g, group_gap = group_gate_pruned(l, m, allowed, n_groups, top_groups)
+        cand = np.isfinite(log_g)
+        idx = np.argsort(np.where(cand, -g, np.inf), axis=1, kind="stable")[:, :k].astype(np.int64)
+    else:
+        g, log_g = group_gate(l, m, allowed, n_groups)
+        idx = topk_route(g, allowed, k)
     w = combine_weights(g, idx, renorm)
     counts, offsets, perm = route_tables(idx, l.shape[1])
     boundary, adjacent = topk_gaps(log_g, idx, allowed)
+    if pruned:
+        boundary = np.minimum(boundary, group_gap)
     return dict(allowed=allowed, l=l, m=m, g=g, log_g=log_g, idx=idx, w=w, counts=counts,
                 offsets=offsets, perm=perm, gap_boundary=boundary, gap_adjacent=adjacent)
 
 
 def layer_forward(inp: Dict[str, np.ndarray], n_groups: int, k: int, act: int, renorm: bool = False,
-                  rows: Optional[Sequence[int]] = None) -> Dict[str, np.ndarray]:
+                  rows: Optional[Sequence[int]] = None, top_groups: int = 0) -> Dict[str, np.ndarray]:
     """The whole MoE-layer forward (Eq. 1 with the Eq. 4-7 gate and the codec).
 
     ``inp`` holds float64 arrays: X, W_local, b_local, W_global, b_global,
@@ -266,11 +345,12 @@ def layer_forward(inp: Dict[str, np.ndarray], n_groups: int, k: int, act: int, r
     The gate sees X; the experts see the decoded X_hat (X when no codec).
     ``rows`` restricts the expert/combine part to those token rows (the gate
     and routing always cover every token, since the histogram needs them all).
+    ``top_groups`` > 0 selects the pruned group gate (``group_gate_pruned``).
     Returns the routing results plus Z, X_hat and y for the chosen rows.
     """
     X = np.asarray(inp["X"], dtype=np.float64)
     r = gate_and_route(X, inp["W_local"], inp["b_local"], inp.get("W_global"), inp.get("b_global"),
-                       inp["mask"], n_groups, k, renorm)
+                       inp["mask"], n_groups, k, renorm, top_groups)
     sel = np.arange(X.shape[0]) if rows is None else np.asarray(rows, dtype=np.int64)
     Xs = X[sel]
     if inp.get("V_enc") is not None:

@@ -24,7 +24,7 @@ GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "wor
 def _num(v):
     if isinstance(v, str):
         return {"ln2": math.log(2.0), "ln3": math.log(3.0), "ln4": math.log(4.0), "ln5": math.log(5.0),
-                "ln3-0.5": math.log(3.0) - 0.5}[v]
+                "ln3-0.5": math.log(3.0) - 0.5, "ln3-ln2": math.log(1.5)}[v]
     return float(v)
 
 
@@ -416,10 +416,104 @@ def pin_layer_rows_subset(orc, seed=13):
     np.testing.assert_allclose(part["y"], full["y"][rows], rtol=1e-13, atol=1e-14)
 
 
+# ----------------------------------------------------------- top-group pruning
+
+def _pruning_example():
+    ex = golden()["group_pruning"]
+    X = np.array(ex["x"])
+    Wl = np.array([[_num(v) for v in row] for row in ex["W_local"]])
+    Wg = np.array([[_num(v) for v in row] for row in ex["W_global"]])
+    return ex, X, Wl, np.array(ex["b_local"]), Wg, np.array(ex["b_global"])
+
+
+def pin_pruning_golden(orc):
+    """Hand-derived g, Top-k, group margins and the rejection of the worked
+    pruning example (closed forms)."""
+    ex, X, Wl, bl, Wg, bg = _pruning_example()
+    K = ex["n_groups"]
+    for case in ex["cases"]:
+        mask = np.array(case["mask"], np.uint8)
+        G = case["top_groups"]
+        r = orc.gate_and_route(X, Wl, bl, Wg, bg, mask, K, 1, top_groups=G)
+        np.testing.assert_allclose(r["g"], case["g"], rtol=0, atol=1e-12)
+        assert r["idx"].tolist() == case["top1"]
+        l, m = orc.gate_logits(X, Wl, bl, Wg, bg)
+        _, _, gap = orc.group_gate_pruned(l, m, mask.astype(bool), K, G)
+        want = [np.inf if v is None else _num(v) for v in case["group_gap"]]
+        np.testing.assert_allclose(gap, want, rtol=0, atol=1e-12)
+        if case["top2"] is None:
+            try:
+                orc.gate_and_route(X, Wl, bl, Wg, bg, mask, K, 2, top_groups=G)
+            except ValueError:
+                pass
+            else:
+                raise AssertionError("k above the kept groups' candidates must be rejected")
+        else:
+            r2 = orc.gate_and_route(X, Wl, bl, Wg, bg, mask, K, 2, top_groups=G)
+            assert r2["idx"].tolist() == case["top2"]
+            np.testing.assert_allclose(r2["w"], np.take_along_axis(np.array(case["g"]), r2["idx"], axis=1),
+                                       rtol=0, atol=1e-12)
+
+
+def pin_pruning_all_groups_is_unpruned(orc, seed=14):
+    """Keeping every live group (top_groups >= live groups) is the unpruned gate."""
+    rng = np.random.default_rng(seed)
+    for (E, K) in [(8, 2), (12, 3), (64, 8)]:
+        X, Wl, bl, Wg, bg = _rand_gate(rng, 30, 16, E, K)
+        mask = (rng.random(E) < 0.6).astype(np.uint8)
+        mask[: E // K] = 0  # one dead group
+        mask[E // K] = 1
+        allowed = mask.astype(bool)
+        l, m = orc.gate_logits(X, Wl, bl, Wg, bg)
+        g0, lg0 = orc.group_gate(l, m, allowed, K)
+        for G in (K - 1, K):
+            g1, lg1, gap = orc.group_gate_pruned(l, m, allowed, K, G)
+            np.testing.assert_allclose(g1, g0, rtol=1e-12, atol=1e-15)
+            assert np.all(np.isinf(gap))
+
+
+def pin_pruning_bruteforce(orc, seed=15):
+    """Per token, the kept groups are the size-G subset of live groups with the
+    largest total p_group (ties to the lexicographically smallest subset), and
+    g is scipy's softmax of m over that subset times scipy's softmax of l over
+    each kept group's allowed members; Top-k is the brute-force best k-subset
+    of the candidates with the lower-index tie rule."""
+    rng = np.random.default_rng(seed)
+    for (E, K, G, k) in [(8, 4, 2, 3), (12, 4, 1, 2), (6, 3, 2, 3)]:
+        T = 40
+        X = rng.integers(-2, 3, size=(T, 3)).astype(np.float64)
+        Wl = rng.integers(-1, 2, size=(E, 3)).astype(np.float64) * 0.5
+        Wg = rng.integers(-1, 2, size=(K, 3)).astype(np.float64) * 0.5
+        bl, bg = np.zeros(E), np.zeros(K)
+        mask = np.ones(E, np.uint8)
+        mask[rng.choice(E, 1)] = 0
+        r = orc.gate_and_route(X, Wl, bl, Wg, bg, mask, K, k, top_groups=G)
+        gsz = E // K
+        live = [j for j in range(K) if mask[j * gsz:(j + 1) * gsz].any()]
+        lx, mx = X @ Wl.T + bl, X @ Wg.T + bg
+        for t in range(T):
+            pg = softmax(mx[t, live])
+            best = max(itertools.combinations(range(len(live)), G),
+                       key=lambda S: (round(float(sum(pg[list(S)])), 12), [-q for q in S]))
+            kept = [live[q] for q in best]
+            pg_kept = softmax(mx[t, kept])
+            want = np.zeros(E)
+            for q, j in enumerate(kept):
+                mem = [i for i in range(j * gsz, (j + 1) * gsz) if mask[i]]
+                want[mem] = pg_kept[q] * softmax(lx[t, mem])
+            np.testing.assert_allclose(r["g"][t], want, rtol=1e-12, atol=1e-15)
+            cand = np.flatnonzero(want > 0)
+            best_sub = min(itertools.combinations(cand.tolist(), k),
+                           key=lambda S: (-round(float(want[list(S)].sum()), 12), S))
+            got = r["idx"][t].tolist()
+            assert sorted(got) == list(best_sub), (t, got, best_sub)
+
+
 ALL_PINS = [
     pin_gate_golden, pin_gate_sums_to_one, pin_masked_never_selected, pin_single_group_is_softmax,
     pin_group_factorisation, pin_topk_bruteforce, pin_rejections, pin_route_golden,
     pin_route_invariants, pin_codec_golden, pin_codec_identity, pin_codec_projection,
     pin_ffn_golden, pin_activations_library, pin_ffn_bruteforce, pin_layer_single_expert,
     pin_layer_linearity, pin_layer_codec_golden, pin_layer_rows_subset, pin_layer_pairing_golden,
+    pin_pruning_golden, pin_pruning_all_groups_is_unpruned, pin_pruning_bruteforce,
 ]

@@ -164,6 +164,61 @@ def m_weights_slot_rolled(g, idx, renorm):
     return np.roll(_combine_weights(g, idx, renorm), 1, axis=1)
 
 
+def _pruned_variant(l, m, allowed, K, G, order="p_group", ties="lower", renorm=True):
+    # group_gate_pruned with one step changed (the ranking key, the tie rule,
+    # or the renormalisation of p_group over the kept groups)
+    T, E = l.shape
+    b = orc.group_bounds(E, K)
+    live = [j for j in range(K) if allowed[b[j]:b[j + 1]].any()]
+    g = np.zeros((T, E))
+    log_g = np.full((T, E), -np.inf)
+    gap = np.full(T, np.inf)
+    for t in range(T):
+        if order == "local":
+            score = [max(l[t, i] for i in range(b[j], b[j + 1]) if allowed[i]) for j in live]
+        elif order == "lowest":
+            score = [-m[t, j] for j in live]
+        else:
+            score = [m[t, j] for j in live]
+        sign = 1 if ties == "lower" else -1
+        ranked = sorted(range(len(live)), key=lambda q: (-score[q], sign * live[q]))
+        kept = sorted(live[q] for q in ranked[:G])
+        if G < len(live):
+            gap[t] = m[t, live[ranked[G - 1]]] - m[t, live[ranked[G]]]
+        pool = kept if renorm else live
+        mk = m[t, pool]
+        lse = mk.max() + np.log(np.exp(mk - mk.max()).sum())
+        for j in kept:
+            mem = [i for i in range(b[j], b[j + 1]) if allowed[i]]
+            z = l[t, mem]
+            lz = z.max() + np.log(np.exp(z - z.max()).sum())
+            for i, zi in zip(mem, z):
+                log_g[t, i] = (m[t, j] - lse) + (zi - lz)
+                g[t, i] = np.exp(log_g[t, i])
+    return g, log_g, gap
+
+
+def m_pruned_no_renorm(l, m, allowed, K, G):
+    return _pruned_variant(l, m, allowed, K, G, renorm=False)
+
+
+def m_pruned_keeps_lowest(l, m, allowed, K, G):
+    return _pruned_variant(l, m, allowed, K, G, order="lowest")
+
+
+def m_pruned_ties_to_higher_group(l, m, allowed, K, G):
+    return _pruned_variant(l, m, allowed, K, G, ties="higher")
+
+
+def m_pruned_by_best_local(l, m, allowed, K, G):
+    return _pruned_variant(l, m, allowed, K, G, order="local")
+
+
+def m_pruning_ignored(l, m, allowed, K, G):
+    g, log_g = orc.group_gate(l, m, allowed, K)
+    return g, log_g, np.full(l.shape[0], np.inf)
+
+
 def m_gap_wrong_sign(log_g, idx, allowed):
     b, a = _topk_gaps(log_g, idx, allowed)
     return -b, a
@@ -190,6 +245,11 @@ MUTANTS = [
     ("layer_forward", m_experts_rolled),
     ("layer_forward", m_slot_weight_shifted),
     ("combine_weights", m_weights_slot_rolled),
+    ("group_gate_pruned", m_pruned_no_renorm),
+    ("group_gate_pruned", m_pruned_keeps_lowest),
+    ("group_gate_pruned", m_pruned_ties_to_higher_group),
+    ("group_gate_pruned", m_pruned_by_best_local),
+    ("group_gate_pruned", m_pruning_ignored),
     ("topk_gaps", m_gap_wrong_sign),
 ]
 
