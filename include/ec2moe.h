@@ -78,13 +78,24 @@ typedef enum ec2moe_act { EC2MOE_GELU = 0, EC2MOE_SWIGLU = 1 } ec2moe_act;
  *  n_shared     always-on shared experts (weight 1, not masked, not counted)
  *  d_ff_shared  hidden width of each shared expert
  *  renorm_topk  0: the combine weight is g_i itself (Eq. 1 with G = g);
- *               1: g_i divided by the sum of g over the token's top-k */
+ *               1: g_i divided by the sum of g over the token's top-k
+ *  top_groups   0: every group takes part (Eq. 5-7).  G >= 1: top-group
+ *               pruning, the group gate evaluated hierarchically -- per token
+ *               only the G live groups (groups with an allowed expert) with
+ *               the largest p_group of Eq. 6 keep their experts (ties to the
+ *               lower group index, decided on the fp32 global logits), and
+ *               p_group is renormalised over them, so the weights of Eq. 7
+ *               still sum to 1 over the candidates.  G at or above the number
+ *               of live groups (or K = 1) prunes nothing.  k above the allowed
+ *               experts of the G live groups with the fewest returns
+ *               EC2MOE_ERR_TOO_FEW_EXPERTS; G < 0 EC2MOE_ERR_INVALID_ARG. */
 typedef struct ec2moe_layer_desc {
   int32_t T, d, E, d_ff, k, n_groups;
   int32_t act, dtype;
   int32_t r;
   int32_t n_shared, d_ff_shared;
   int32_t renorm_topk;
+  int32_t top_groups;
 } ec2moe_layer_desc;
 
 /* Weights of one layer (device pointers, NULL where absent).

@@ -147,6 +147,7 @@ ec2moe_status check_desc(const ec2moe_layer_desc* d) {
   if (d->dtype != EC2MOE_F32 && d->dtype != EC2MOE_BF16) return EC2MOE_ERR_INVALID_ARG;
   if (d->act != EC2MOE_GELU && d->act != EC2MOE_SWIGLU) return EC2MOE_ERR_INVALID_ARG;
   if (d->renorm_topk != 0 && d->renorm_topk != 1) return EC2MOE_ERR_INVALID_ARG;
+  if (d->top_groups < 0) return EC2MOE_ERR_INVALID_ARG;
   if (d->E % d->n_groups != 0) return EC2MOE_ERR_INVALID_ARG;
   if (d->k > d->E) return EC2MOE_ERR_TOO_FEW_EXPERTS;
   if (d->E > EC2MOE_MAX_EXPERTS || d->n_groups > EC2MOE_MAX_GROUPS || d->k > EC2MOE_MAX_TOPK ||
@@ -184,6 +185,29 @@ ec2moe_status check_mask(const ec2moe_layer_desc* d, const uint8_t* mask, uint32
     }
   if (n == 0) return EC2MOE_ERR_ALL_MASKED;
   if (n < d->k) return EC2MOE_ERR_TOO_FEW_EXPERTS;
+  if (d->top_groups > 0 && d->n_groups > 1) {
+    // top-group pruning: the G live groups with the fewest allowed experts
+    // must still hold k candidates
+    int sizes[EC2MOE_MAX_GROUPS];
+    int live = 0;
+    const int gsize = d->E / d->n_groups;
+    for (int g = 0; g < d->n_groups; ++g) {
+      int c = 0;
+      for (int e = g * gsize; e < (g + 1) * gsize; ++e) c += mask[e] ? 1 : 0;
+      if (c > 0) sizes[live++] = c;
+    }
+    if (d->top_groups < live) {
+      for (int i = 1; i < live; ++i)
+        for (int j = i; j > 0 && sizes[j] < sizes[j - 1]; --j) {
+          const int t = sizes[j];
+          sizes[j] = sizes[j - 1];
+          sizes[j - 1] = t;
+        }
+      int floor_k = 0;
+      for (int i = 0; i < d->top_groups; ++i) floor_k += sizes[i];
+      if (floor_k < d->k) return EC2MOE_ERR_TOO_FEW_EXPERTS;
+    }
+  }
   return EC2MOE_OK;
 }
 
@@ -562,6 +586,7 @@ ec2moe_status ec2moe_gate(const ec2moe_layer_desc* desc, const void* X, const fl
   a.K = desc->n_groups;
   a.k = desc->k;
   a.renorm = desc->renorm_topk;
+  a.top_groups = desc->top_groups;
   a.topk_idx = topk_idx;
   a.topk_w = topk_w;
   EC2MOE_CUDA(launch_gate(a, is_bf16(desc), stream));
@@ -743,6 +768,7 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   ga.K = desc->n_groups;
   ga.k = desc->k;
   ga.renorm = desc->renorm_topk;
+  ga.top_groups = desc->top_groups;
   ga.topk_idx = topk_idx;
   ga.topk_w = topk_w;
   // bf16 layers route inside the gate kernel (per-tile row reservations); the
@@ -910,6 +936,7 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
     ga.K = sub.n_groups;
     ga.k = sub.k;
     ga.renorm = sub.renorm_topk;
+    ga.top_groups = sub.top_groups;
     ga.topk_idx = idx_i;
     ga.topk_w = tw_i;
     if (bf) {

@@ -15,6 +15,12 @@
 // itself.  Top-k takes the largest score, ties to the lower index, k times.
 // The combine weight is g_i = exp((m_k - LSE_m) + (l_i - lse_k)) where LSE_m is
 // the log-sum-exp of m over groups with at least one allowed expert.
+//
+// Top-group pruning (top_groups = G > 0): before the scores, each token keeps
+// only the G live groups with the largest global logit m_k (the order of
+// p_group; ties to the lower group index); the other groups are treated as if
+// they had no allowed expert, so their experts are not candidates and LSE_m
+// runs over the kept groups (p_group renormalised over them).
 #include <stdlib.h>
 
 #include <cuda_bf16.h>
@@ -167,6 +173,22 @@ __global__ void __launch_bounds__(WARPS * 32) gate_topk_kernel(const KParams p) 
         G[16 + lane] = live ? 1.0f : 0.0f;
       }
       __syncwarp();
+      // ---- top-group pruning: only the top_groups live groups by m stay live
+      if (nglob && p.top_groups > 0 && p.top_groups < p.K) {
+        bool keep = false;
+        if (lane < p.K && G[16 + lane] != 0.0f) {
+          const float mg = L[p.E + lane];
+          int rank = 0;
+          for (int j = 0; j < p.K; ++j) {
+            const float mj = L[p.E + j];
+            if (j != lane && G[16 + j] != 0.0f && (mj > mg || (mj == mg && j < lane))) ++rank;
+          }
+          keep = rank < p.top_groups;
+        }
+        __syncwarp();
+        if (lane < p.K) G[16 + lane] = keep ? 1.0f : 0.0f;
+        __syncwarp();
+      }
       // ---- log-sum-exp of the global logits over live groups (Eq. 6)
       float lse_m = 0.0f;
       if (nglob) {
@@ -189,9 +211,11 @@ __global__ void __launch_bounds__(WARPS * 32) gate_topk_kernel(const KParams p) 
           const int grp = e / gsize;
           const float le = L[e];
           if (nglob) {
-            const float mk = L[p.E + grp];
-            key[i] = (mk - G[grp]) + le;
-            lw[i] = (mk - lse_m) + (le - G[grp]);
+            if (G[16 + grp] != 0.0f) {  // a kept group
+              const float mk = L[p.E + grp];
+              key[i] = (mk - G[grp]) + le;
+              lw[i] = (mk - lse_m) + (le - G[grp]);
+            }
           } else {
             key[i] = le;
             lw[i] = le - G[0];
@@ -305,7 +329,25 @@ __device__ void decide_token_warp(const KParams& p, const float* L, int tok, int
         if (allowed_bit(p, e)) sum += expf(L[e] - mx);
       if (mx > -CUDART_INF_F) lse_mine = mx + logf(sum);
     }
-    const float mk_mine = (lane < p.K && lse_mine > -CUDART_INF_F) ? L[p.E + lane] : -CUDART_INF_F;
+    // groups that stay: the live ones, or with top-group pruning the
+    // top_groups live ones by m (ties to the lower group index)
+    unsigned kept = __ballot_sync(0xffffffffu, lane < p.K && lse_mine > -CUDART_INF_F);
+    if (p.top_groups > 0 && p.top_groups < p.K) {
+      bool keep = false;
+      if ((kept >> lane) & 1u) {
+        const float mg = L[p.E + lane];
+        int rank = 0;
+        for (int j = 0; j < p.K; ++j)
+          if (j != lane && ((kept >> j) & 1u)) {
+            const float mj = L[p.E + j];
+            rank += (mj > mg || (mj == mg && j < lane)) ? 1 : 0;
+          }
+        keep = rank < p.top_groups;
+      }
+      kept = __ballot_sync(0xffffffffu, keep);
+      if (!keep) lse_mine = -CUDART_INF_F;
+    }
+    const float mk_mine = ((kept >> lane) & 1u) ? L[p.E + lane] : -CUDART_INF_F;
     float mxm = mk_mine;
 #pragma unroll
     for (int sh = 16; sh > 0; sh >>= 1) mxm = fmaxf(mxm, __shfl_xor_sync(0xffffffffu, mxm, sh));
@@ -319,7 +361,7 @@ __device__ void decide_token_warp(const KParams& p, const float* L, int tok, int
       const int g = (e < p.E ? e : 0) / gsize;
       const float lse_g = __shfl_sync(0xffffffffu, lse_mine, g);
       const float mk = L[p.E + (g < p.K ? g : 0)];
-      key[i] = al[i] ? (mk - lse_g) + lv[i] : -CUDART_INF_F;
+      key[i] = (al[i] && ((kept >> g) & 1u)) ? (mk - lse_g) + lv[i] : -CUDART_INF_F;
       lw[i] = (mk - lse_m) + (lv[i] - lse_g);
     }
   }
@@ -861,6 +903,7 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* rout
   p.K = a.K;
   p.k = a.k;
   p.renorm = a.renorm;
+  p.top_groups = a.top_groups;
   p.topk_idx = a.topk_idx;
   p.topk_w = a.topk_w;
   p.route_counts = nullptr;

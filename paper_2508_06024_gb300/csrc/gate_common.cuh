@@ -21,6 +21,7 @@ struct KParams {
   const float* b_global;
   uint32_t mask_bits[4];
   int T, d, E, K, k, renorm;
+  int top_groups;  // > 0 and < live groups: per token only the top_groups groups by m keep their experts
   int32_t* topk_idx;
   float* topk_w;
   int32_t* route_counts;  // fused routing: per-expert row counters (zero at launch); nullptr = gate only

@@ -93,9 +93,10 @@ struct GcParams {
 // One token's decision by one thread, from its logits row L[0..E) (local),
 // L[E..E+K) (global) and a scratch row G[0..K) -- the arithmetic of
 // decide_token_warp with sequential sums: per-group log-sum-exp over the
-// allowed members (Eq. 5), log-sum-exp of the global logits over live groups
-// (Eq. 6), key = (m_g - lse_g) + l_i (K = 1: l_i), weight exp((m_g - LSE_m) +
-// (l_i - lse_g)) (Eq. 7); Top-k by insertion into a sorted list (larger key
+// allowed members (Eq. 5), top-group pruning when top_groups > 0 (only the
+// top_groups live groups by m stay), log-sum-exp of the global logits over the
+// live (kept) groups (Eq. 6), key = (m_g - lse_g) + l_i (K = 1: l_i), weight
+// exp((m_g - LSE_m) + (l_i - lse_g)) (Eq. 7); Top-k by insertion into a sorted list (larger key
 // first, ties to the lower index).  Slots left empty by non-finite keys take
 // the lowest allowed experts not chosen yet.  The mask words are in
 // registers, so the loads of one pass are independent of each other.
@@ -129,8 +130,8 @@ __device__ __forceinline__ void topk_insert(float* tk, float* tl, int* ti, float
 
 // KS >= k slots are kept (KS in {1, 2, 4, 8}).
 template <int KS>
-__device__ void decide_token_thread(int E, int K, int k, int renorm, const MaskRegs m, const float* L, float* G,
-                                    int32_t* topk_idx, float* topk_w, int tok, int* s_idx) {
+__device__ void decide_token_thread(int E, int K, int k, int renorm, int top_groups, const MaskRegs m, const float* L,
+                                    float* G, int32_t* topk_idx, float* topk_w, int tok, int* s_idx) {
   const bool grouped = K > 1;
   const int ng = grouped ? K : 1;
   const int gsize = E / ng;
@@ -173,10 +174,31 @@ __device__ void decide_token_thread(int E, int K, int k, int renorm, const MaskR
 #pragma unroll 4
       for (int e = lo; e < hi; ++e)
         if (m.has(e)) sum += expf(L[e] - mx);
-      const float lse = mx > -CUDART_INF_F ? mx + logf(sum) : -CUDART_INF_F;
-      G[g] = lse;
-      if (lse > -CUDART_INF_F) mxm = fmaxf(mxm, L[E + g]);
+      G[g] = mx > -CUDART_INF_F ? mx + logf(sum) : -CUDART_INF_F;
     }
+    // top-group pruning: only the top_groups live groups by m (ties to the
+    // lower group index) keep their experts and their share of p_group
+    if (top_groups > 0 && top_groups < ng) {
+      uint32_t keep = 0;
+#pragma unroll 1
+      for (int g = 0; g < ng; ++g) {
+        if (G[g] == -CUDART_INF_F) continue;
+        const float mg = L[E + g];
+        int rank = 0;
+#pragma unroll 1
+        for (int j = 0; j < ng; ++j) {
+          const float mj = L[E + j];
+          if (j != g && G[j] > -CUDART_INF_F && (mj > mg || (mj == mg && j < g))) ++rank;
+        }
+        if (rank < top_groups) keep |= 1u << g;
+      }
+#pragma unroll 1
+      for (int g = 0; g < ng; ++g)
+        if (!((keep >> g) & 1u)) G[g] = -CUDART_INF_F;
+    }
+#pragma unroll 1
+    for (int g = 0; g < ng; ++g)
+      if (G[g] > -CUDART_INF_F) mxm = fmaxf(mxm, L[E + g]);
     float summ = 0.0f;
 #pragma unroll 1
     for (int g = 0; g < K; ++g)
@@ -185,6 +207,7 @@ __device__ void decide_token_thread(int E, int K, int k, int renorm, const MaskR
 #pragma unroll 1
     for (int g = 0; g < ng; ++g) {
       const float lg = G[g];
+      if (lg == -CUDART_INF_F) continue;  // no allowed member, or pruned
       const float mk = L[E + g];
       const int lo = g * gsize, hi = lo + gsize;
 #pragma unroll 2
@@ -644,10 +667,10 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
               if (o < O) Lrow[o] = acc[b][j];
             }
           if (tok < p.T) {
-            if (p.k == 1) decide_token_thread<1>(p.E, p.K, p.k, p.renorm, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
-            else if (p.k == 2) decide_token_thread<2>(p.E, p.K, p.k, p.renorm, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
-            else if (p.k <= 4) decide_token_thread<4>(p.E, p.K, p.k, p.renorm, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
-            else decide_token_thread<8>(p.E, p.K, p.k, p.renorm, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+            if (p.k == 1) decide_token_thread<1>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+            else if (p.k == 2) decide_token_thread<2>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+            else if (p.k <= 4) decide_token_thread<4>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+            else decide_token_thread<8>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
           }
         }
       } else if (!PREP) {

@@ -70,6 +70,7 @@ struct GateArgs {
   const float* b_global;
   uint32_t mask_bits[4];  // bit e = expert e allowed (E <= 128)
   int T, d, E, K, k, renorm;
+  int top_groups;  // > 0: keep only that many live groups per token (top-group pruning)
   int32_t* topk_idx;
   float* topk_w;
   // Routing fused into the gate (layer path; both nullptr: gate only): the

@@ -22,6 +22,19 @@
 // accumulators (tmem_full/tmem_empty) so the epilogue of tile i overlaps the
 // main loop of tile i+1.
 //
+// CTA pairs (PAIR): a cluster of two CTAs on two SMs computes one 256-row tile
+// with tcgen05.mma.cta_group::2 (M = 256).  Each CTA stages its own 128 rows
+// of A and its half of the B tile (for SwiGLU: the even CTA the W1 rows, the
+// odd one the W3 rows), so a CTA moves 2/3 of the operand bytes per k-block of
+// an unpaired 128 x 256 tile and the same shared memory holds 1.5x the stages.
+// The even CTA issues the MMAs; the odd CTA's MMA warp relays "stage s has
+// landed" from its own full barrier to the even CTA (remote mbarrier arrive),
+// so each CTA's copies complete on its own barriers and each can drain its own
+// copies after an abort.  MMA completion is committed to both CTAs' empty and
+// accumulator-full barriers (multicast); both CTAs' epilogue warps release an
+// accumulator on the even CTA's tmem_empty barrier.  TMEM is allocated for the
+// pair (cta_group::2), and a cluster barrier precedes its release.
+//
 // Every mbarrier wait is bounded by a clock64 budget.  A wait that gives up
 // sets the device error word, raises a CTA-wide abort flag that ends every
 // other wait at once, waits (again bounded) for the CTA's own TMA copies and
@@ -33,7 +46,10 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <stdlib.h>
+
 #include <atomic>
+#include <cmath>
 #include <mutex>
 
 #include "common.cuh"
@@ -94,10 +110,12 @@ __device__ __forceinline__ TileCoord decode_tile(int tile, const int* tile_prefi
 
 constexpr int pow2_at_least(int x) { return x <= 32 ? 32 : (x <= 64 ? 64 : (x <= 128 ? 128 : (x <= 256 ? 256 : 512))); }
 
-template <int BN, int EPI, int STAGES>
+template <int BN, int EPI, int STAGES, bool PAIR>
 struct Cfg {
+  static constexpr int CTA_B_ROWS = PAIR ? BN / 2 : BN;  // rows of the B tile this CTA stages
+  static constexpr int TILE_M = PAIR ? 2 * BM : BM;      // rows of one (pair) tile
   static constexpr int A_BYTES = BM * BK * 2;
-  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int B_BYTES = CTA_B_ROWS * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int BN_OUT = (EPI == EPI_SWIGLU) ? BN / 2 : BN;
   // columns of a tile split among the warps of a lane quadrant: PARTS parts
@@ -107,7 +125,8 @@ struct Cfg {
   static constexpr int CW = 16;  // columns per TMEM load
   static_assert(PART % CW == 0, "epilogue chunks must tile each part exactly");
   static constexpr int TMEM_COLS = pow2_at_least(2 * BN);  // two accumulators
-  static constexpr int BAR_BYTES = (2 * STAGES + 5) * 8;
+  // mbarriers: full[S], empty[S], (PAIR) ready[S], tmem_full[2], tmem_empty[2], drain
+  static constexpr int N_BARS = (PAIR ? 3 : 2) * STAGES + 5;
   static constexpr int STG_PITCH = CW * 2 + 16;          // bytes per staged row (padded)
   // Row-segment epilogue (contiguous or per-row destinations): the four warps
   // of a lane quadrant stage 32 rows x 64 columns (bf16, 128-byte rows,
@@ -120,35 +139,50 @@ struct Cfg {
   static constexpr int STG_BYTES =
       ROWSEG ? 4 * 32 * SLAB * 2 : (EPI == EPI_PARTIAL ? 0 : EPI_WARPS * 32 * STG_PITCH);
   static constexpr int OFF_INTS = 132;  // expert offsets of EPI_REPLICATE's relative mode (<= 128 + 1, padded)
-  static constexpr int SMEM = 1024 + STAGES * STAGE_BYTES + BAR_BYTES + 16 + 2 * (MAX_GROUPS + 1) * 4 + OFF_INTS * 4 +
-                              STG_BYTES;
+  // byte offsets from the 1024-aligned base: operand stages, barriers, TMEM
+  // slot + abort flag (16 bytes), tile prefix, group first rows, expert
+  // offsets, then the epilogue staging (128-byte aligned: its rows are
+  // written with 16-byte vector stores)
+  static constexpr int OFF_BARS = STAGES * STAGE_BYTES;
+  static constexpr int OFF_SLOT = OFF_BARS + N_BARS * 8;
+  static constexpr int OFF_PREFIX = OFF_SLOT + 16;
+  static constexpr int OFF_ROW0 = OFF_PREFIX + (MAX_GROUPS + 1) * 4;
+  static constexpr int OFF_SOFF = OFF_ROW0 + (MAX_GROUPS + 1) * 4;
+  static constexpr int OFF_STG = (OFF_SOFF + OFF_INTS * 4 + 127) / 128 * 128;
+  static constexpr int SMEM = 1024 + OFF_STG + STG_BYTES;
+  static_assert(OFF_BARS % 8 == 0 && OFF_STG % 128 == 0, "shared memory alignment");
   static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
-template <int BN, int EPI, int STAGES>
+template <int BN, int EPI, int STAGES, bool PAIR>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmB2, const Params p) {
-  using C = Cfg<BN, EPI, STAGES>;
+  using C = Cfg<BN, EPI, STAGES, PAIR>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * C::A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BARS);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
-  uint64_t* tfull = bars + 2 * STAGES;
-  uint64_t* tempty = bars + 2 * STAGES + 2;
-  uint64_t* drain = bars + 2 * STAGES + 4;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * STAGES + 5);
+  uint64_t* ready = bars + 2 * STAGES;  // PAIR, even CTA: the odd CTA's stage s has landed
+  uint64_t* tfull = bars + (PAIR ? 3 : 2) * STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tfull + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_SLOT);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  int* tile_prefix = reinterpret_cast<int*>(tmem_slot + 4);
-  int* row0 = tile_prefix + (MAX_GROUPS + 1);
-  int* s_off = row0 + MAX_GROUPS + 1;                                    // [C::OFF_INTS]
-  uint8_t* stg_all = reinterpret_cast<uint8_t*>(s_off + C::OFF_INTS);  // epilogue staging, 16-byte aligned
+  int* tile_prefix = reinterpret_cast<int*>(smem + C::OFF_PREFIX);
+  int* row0 = reinterpret_cast<int*>(smem + C::OFF_ROW0);
+  int* s_off = reinterpret_cast<int*>(smem + C::OFF_SOFF);  // [C::OFF_INTS]
+  uint8_t* stg_all = smem + C::OFF_STG;                      // epilogue staging
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  // PAIR: rank in the CTA pair (0 issues the MMAs), the pair's tile stream
+  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  const int tile_first = PAIR ? static_cast<int>(cluster_id_x()) : static_cast<int>(blockIdx.x);
+  const int tile_step = PAIR ? static_cast<int>(cluster_count_x()) : static_cast<int>(gridDim.x);
   // Barrier set-up, TMEM allocation and descriptor prefetch overlap the
   // previous kernel; everything that reads its results comes after pdl_wait.
   pdl_trigger();
@@ -157,10 +191,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
       mbar_init(smem_u32(&empty[s]), 1);
+      if (PAIR) mbar_init(smem_u32(&ready[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
-      mbar_init(smem_u32(&tempty[a]), EPI_WARPS);
+      mbar_init(smem_u32(&tempty[a]), PAIR ? 2 * EPI_WARPS : EPI_WARPS);
     }
     mbar_init(smem_u32(drain), 1);
     *abort_flag = 0;
@@ -179,7 +214,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             mg = p.offsets[g + 1] - r0;
           }
           row0[g] = r0;
-          return (mg + BM - 1) / BM;
+          return (mg + C::TILE_M - 1) / C::TILE_M;
         },
         tile_prefix);
     if (EPI == EPI_REPLICATE && p.rep_counts)
@@ -192,13 +227,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (EPI == EPI_SWIGLU) tma_prefetch_desc(&tmB2);
   }
   if (warp == 1) {
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                 "r"(C::TMEM_COLS)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    if (PAIR) {
+      // the pair's columns, allocated by one warp of each CTA together
+      asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                   "r"(C::TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    } else {
+      asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                   "r"(C::TMEM_COLS)
+                   : "memory");
+      asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
   }
   tc_fence_before();
   __syncthreads();
+  // PAIR: both CTAs' barriers are initialised before either arrives remotely
+  if (PAIR) cluster_sync_all();
   tc_fence_after();
   pdl_wait();
   const uint32_t tmem_base = *tmem_slot;
@@ -217,10 +262,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t issued_phase = 0;
       int cursor = 0;
       bool ok = true;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+      for (int tile = tile_first; tile < n_tiles && ok; tile += tile_step) {
         const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
         const int a_row = static_cast<int>(p.a_row_base) + (p.offsets ? row0[tc.g] : (p.a_shared ? 0 : row0[tc.g])) +
-                          tc.m_blk * BM;
+                          tc.m_blk * C::TILE_M + static_cast<int>(rank) * BM;
         const int b_row = tc.g * p.b_group_rows + tc.n_blk * C::BN_OUT;
         const int kb0 = (tile % p.split_k) * p.kb_per_split;
         const int kb1 = kb0 + p.kb_per_split < num_kb ? kb0 + p.kb_per_split : num_kb;
@@ -232,11 +277,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           const uint32_t fb = smem_u32(&full[stage]);
           mbar_expect_tx(fb, C::STAGE_BYTES);
           tma_load_2d(smem_u32(sA + stage * C::A_BYTES), &tmA, kb * BK, a_row, fb);
-          if (EPI == EPI_SWIGLU) {
+          if (EPI == EPI_SWIGLU && PAIR) {
+            // the even CTA stages the W1 rows of the tile, the odd CTA the W3 rows
+            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), rank ? &tmB2 : &tmB, kb * BK, b_row, fb);
+          } else if (EPI == EPI_SWIGLU) {
             tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK, b_row, fb);
             tma_load_2d(smem_u32(sB + stage * C::B_BYTES + C::B_BYTES / 2), &tmB2, kb * BK, b_row, fb);
           } else {
-            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK, b_row, fb);
+            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK,
+                        b_row + static_cast<int>(rank) * C::CTA_B_ROWS, fb);
           }
           issued |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -253,9 +302,33 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
     }
   } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t IDESC = idesc_bf16(BM, BN);
+    if (PAIR && rank != 0) {
+      // ------------------------------------------------ odd CTA of a pair: relay
+      // Each stage of this CTA that has landed is announced to the even CTA,
+      // whose MMAs read it.
+      if (lane == 0) {
+        int stage = 0;
+        uint32_t phase = 0;
+        int cursor = 0;
+        bool ok = true;
+        for (int tile = tile_first; tile < n_tiles && ok; tile += tile_step) {
+          (void)decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
+          for (int kb = 0; kb < num_kb; ++kb) {
+            if (!mbar_wait(smem_u32(&full[stage]), phase, budget, abort_flag, &g_tc_error)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_remote(map_to_rank(smem_u32(&ready[stage]), 0));
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+    } else if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      constexpr uint32_t IDESC = idesc_bf16(C::TILE_M, BN);
       constexpr uint64_t DA_STAGE = C::A_BYTES >> 4;
       constexpr uint64_t DB_STAGE = C::B_BYTES >> 4;
       const uint64_t da0 = sdesc_sw128(smem_u32(sA));
@@ -267,13 +340,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int it = 0;
       int cursor = 0;
       bool ok = true, any = false;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++it) {
+      for (int tile = tile_first; tile < n_tiles && ok; tile += tile_step, ++it) {
         (void)decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
         const int kb0 = (tile % p.split_k) * p.kb_per_split;
         const int kb1 = kb0 + p.kb_per_split < num_kb ? kb0 + p.kb_per_split : num_kb;
         const int acc = it & 1;
         const uint32_t acc_phase = (it >> 1) & 1;
-        if (!mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, budget, abort_flag, &g_tc_error)) {
+        // PAIR: the odd CTA's epilogue warps release the accumulator remotely
+        const bool freed = PAIR ? mbar_wait_cluster(smem_u32(&tempty[acc]), acc_phase ^ 1u, budget, abort_flag, &g_tc_error)
+                                : mbar_wait(smem_u32(&tempty[acc]), acc_phase ^ 1u, budget, abort_flag, &g_tc_error);
+        if (!freed) {
           ok = false;
           break;
         }
@@ -284,6 +360,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             ok = false;
             break;
           }
+          if (PAIR && !mbar_wait_cluster(smem_u32(&ready[stage]), phase, budget, abort_flag, &g_tc_error)) {
+            ok = false;
+            break;
+          }
           tc_fence_after();
           // Descriptors of this stage: the stage-0 descriptors plus the stage
           // offset; each K = 16 step adds 32 bytes (2 in the address field).
@@ -291,22 +371,31 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           // below 256 KB.
           const uint64_t da = da0 + static_cast<uint64_t>(stage) * DA_STAGE;
           const uint64_t db = db0 + static_cast<uint64_t>(stage) * DB_STAGE;
-          umma_bf16(d_tmem, da, db, IDESC, kb != kb0 ? 1u : 0u);
+          if (PAIR) {
+            umma_bf16_pair(d_tmem, da, db, IDESC, kb != kb0 ? 1u : 0u);
 #pragma unroll
-          for (int kk = 1; kk < BK / UK; ++kk) umma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, IDESC, 1u);
+            for (int kk = 1; kk < BK / UK; ++kk) umma_bf16_pair(d_tmem, da + 2 * kk, db + 2 * kk, IDESC, 1u);
+          } else {
+            umma_bf16(d_tmem, da, db, IDESC, kb != kb0 ? 1u : 0u);
+#pragma unroll
+            for (int kk = 1; kk < BK / UK; ++kk) umma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, IDESC, 1u);
+          }
           any = true;
-          umma_commit(empty0 + 8u * stage);
+          if (PAIR) umma_commit_pair_mc(empty0 + 8u * stage);
+          else umma_commit(empty0 + 8u * stage);
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1u;
           }
         }
         if (!ok) break;
-        umma_commit(smem_u32(&tfull[acc]));
+        if (PAIR) umma_commit_pair_mc(smem_u32(&tfull[acc]));
+        else umma_commit(smem_u32(&tfull[acc]));
       }
       if ((!ok || *abort_flag) && any) {
         // All MMAs issued so far must finish before TMEM is freed.
-        umma_commit(smem_u32(drain));
+        if (PAIR) umma_commit_pair(smem_u32(drain));
+        else umma_commit(smem_u32(drain));
         mbar_drain(smem_u32(drain), 0, DRAIN_CYCLES);
       }
     }
@@ -317,7 +406,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int row_in_tile = q * 32 + lane;
     int it = 0;
     int cursor = 0;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x, ++it) {
+    for (int tile = tile_first; tile < n_tiles; tile += tile_step, ++it) {
       const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
       const int ks = tile % p.split_k;
       (void)ks;
@@ -325,7 +414,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const uint32_t acc_phase = (it >> 1) & 1;
       // Row metadata first: its global loads overlap the tile's main loop.
       const int mg = p.offsets ? (p.offsets[tc.g + 1] - p.offsets[tc.g]) : p.M;
-      const int local = tc.m_blk * BM + row_in_tile;
+      const int local = tc.m_blk * C::TILE_M + static_cast<int>(rank) * BM + row_in_tile;
       const bool valid = local < mg;
       const long long out_row = p.out_row_base + row0[tc.g] + local;
       long long dest = out_row;
@@ -411,7 +500,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+        if (lane == 0) {
+          // PAIR: both CTAs release the accumulator on the even CTA's barrier
+          if (PAIR) mbar_arrive_remote(map_to_rank(smem_u32(&tempty[acc]), 0));
+          else mbar_arrive(smem_u32(&tempty[acc]));
+        }
         continue;
       }
       // Each chunk of 32 rows x CW columns is staged in shared memory (thread =
@@ -496,16 +589,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&tempty[acc]));
+      if (lane == 0) {
+        if (PAIR) mbar_arrive_remote(map_to_rank(smem_u32(&tempty[acc]), 0));
+        else mbar_arrive(smem_u32(&tempty[acc]));
+      }
     }
   }
 
   tc_fence_before();
   __syncthreads();
+  // PAIR: the even CTA's MMAs write both CTAs' TMEM; neither releases its
+  // columns before both are done with them
+  if (PAIR) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(C::TMEM_COLS)
-                 : "memory");
+    if (PAIR)
+      asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(C::TMEM_COLS)
+                   : "memory");
+    else
+      asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(C::TMEM_COLS)
+                   : "memory");
   }
 }
 
@@ -601,13 +704,69 @@ const char* kernel_name(int epi) {
   }
 }
 
-template <int BN, int EPI, int STAGES>
+// Clusters of two CTAs of `kernel` that fit on the device at once (cached per
+// device and kernel); 0 when the query fails.
+int max_pair_clusters(const void* kernel, int smem) {
+  struct Entry {
+    int dev;
+    const void* kernel;
+    int n;
+  };
+  static std::mutex mu;
+  static Entry cache[32];
+  static int used = 0;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  for (int i = 0; i < used; ++i)
+    if (cache[i].dev == dev && cache[i].kernel == kernel) return cache[i].n;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(2 * sm_count());
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, kernel, &cfg) != cudaSuccess) {
+    (void)cudaGetLastError();
+    n = 0;
+  }
+  if (used < 32) cache[used++] = Entry{dev, kernel, n};
+  return n;
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, size_t smem, cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(2 * clusters);
+  cfg.blockDim = dim3(NUM_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = next_launch_pdl() ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+template <int BN, int EPI, int STAGES, bool PAIR = false>
 cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
-  using C = Cfg<BN, EPI, STAGES>;
-  cudaError_t attr_err = ensure_smem_attr(reinterpret_cast<const void*>(tc_gemm_kernel<BN, EPI, STAGES>), C::SMEM);
+  using C = Cfg<BN, EPI, STAGES, PAIR>;
+  const void* kfn = reinterpret_cast<const void*>(tc_gemm_kernel<BN, EPI, STAGES, PAIR>);
+  cudaError_t attr_err = ensure_smem_attr(kfn, C::SMEM);
   if (attr_err != cudaSuccess) return attr_err;
   CUtensorMap mA, mB, mB2;
-  const int b_box = (EPI == EPI_SWIGLU) ? BN / 2 : BN;
+  const int b_box = (EPI == EPI_SWIGLU || PAIR) ? BN / 2 : BN;
   if (!make_map(&mA, a.A, a.a_rows, a.K, BM)) return cudaErrorInvalidValue;
   if (!make_map(&mB, a.B, a.b_rows, a.K, b_box)) return cudaErrorInvalidValue;
   if (EPI == EPI_SWIGLU) {
@@ -646,22 +805,41 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   }
   p.partial = a.partial;
   p.part_rows = a.part_rows;
-  const long long m_tiles_max = a.max_rows / BM + a.G;
+  const long long m_tiles_max = a.max_rows / C::TILE_M + a.G;
   long long tiles = m_tiles_max * p.n_tiles_n * p.split_k;
+  if (PAIR) {
+    int clusters = max_pair_clusters(kfn, C::SMEM);
+    if (clusters < 1) return cudaErrorInvalidConfiguration;
+    if (tiles < clusters) clusters = static_cast<int>(tiles < 1 ? 1 : tiles);
+    KernelScope ks(a.name ? a.name : kernel_name(EPI), s);
+    cudaError_t le = launch_pairs(tc_gemm_kernel<BN, EPI, STAGES, PAIR>, clusters, (size_t)C::SMEM, s, mA, mB, mB2, p);
+    if (le != cudaSuccess) return le;
+    return cudaGetLastError();
+  }
   int grid = static_cast<int>(tiles < sm_count() ? tiles : sm_count());
   if (grid < 1) grid = 1;
   KernelScope ks(a.name ? a.name : kernel_name(EPI), s);
-  cudaError_t le = launch_kernel(tc_gemm_kernel<BN, EPI, STAGES>, dim3(grid), dim3(NUM_THREADS), (size_t)C::SMEM, s, mA,
-                                 mB, mB2, p);
+  cudaError_t le = launch_kernel(tc_gemm_kernel<BN, EPI, STAGES, PAIR>, dim3(grid), dim3(NUM_THREADS), (size_t)C::SMEM,
+                                 s, mA, mB, mB2, p);
   if (le != cudaSuccess) return le;
   return cudaGetLastError();
 }
 
-// Smem budget of the operand pipeline: as many stages as fit in ~200 KB.
-constexpr int stages_for(int bn) { return (200 * 1024) / (BM * BK * 2 + bn * BK * 2) > 8 ? 8 : (200 * 1024) / (BM * BK * 2 + bn * BK * 2); }
+// Smem budget of the operand pipeline: as many stages as fit in ~200 KB
+// (b_rows: rows of the B tile one CTA stages).
+constexpr int stages_for(int b_rows) {
+  return (200 * 1024) / (BM * BK * 2 + b_rows * BK * 2) > 8 ? 8 : (200 * 1024) / (BM * BK * 2 + b_rows * BK * 2);
+}
 
 template <int EPI>
-cudaError_t launch_epi(const GemmArgs& a, int bn, cudaStream_t s) {
+cudaError_t launch_epi(const GemmArgs& a, int bn, bool pair, cudaStream_t s) {
+  if (pair) {
+    if constexpr (EPI == EPI_STORE || EPI == EPI_GELU || EPI == EPI_SWIGLU || EPI == EPI_SCATTER) {
+      if (bn == 256) return launch_cfg<256, EPI, stages_for(128), true>(a, s);
+      if (bn == 128) return launch_cfg<128, EPI, stages_for(64), true>(a, s);
+    }
+    return cudaErrorInvalidValue;
+  }
   switch (bn) {
     case 32:
       if constexpr (EPI != EPI_SWIGLU) return launch_cfg<32, EPI, stages_for(32)>(a, s);
@@ -675,20 +853,22 @@ cudaError_t launch_epi(const GemmArgs& a, int bn, cudaStream_t s) {
 }
 
 // N-tile choice.  Each candidate is scored by its wave efficiency (tiles over
-// whole waves of one tile per SM) times a per-tile efficiency that falls with
-// the tile width (narrow tiles move more operand bytes per FLOP).  The m-tile
-// count of a grouped GEMM is only known on the device; half a partial tile
-// per group is expected.
-int choose_bn(const GemmArgs& a, int epi) {
+// whole waves of one tile per SM, or per CTA pair) times a per-tile efficiency
+// that falls with the tile width (narrow tiles move more operand bytes per
+// FLOP).  The m-tile count of a grouped GEMM is only known on the device; half
+// a partial tile per group is expected.
+int choose_bn(const GemmArgs& a, int epi, bool pair = false) {
   const int ga = a.g_active > 0 ? a.g_active : a.G;
-  const double m_tiles = (double)a.max_rows / BM + (a.G > 1 ? 0.5 * ga : 0.0) + (a.G == 1 && a.max_rows % BM ? 1 : 0);
-  const int sms = sm_count();
+  const int tm = pair ? 2 * BM : BM;
+  const double m_tiles = (double)a.max_rows / tm + (a.G > 1 ? 0.5 * ga : 0.0) + (a.G == 1 && a.max_rows % tm ? 1 : 0);
+  const int sms = pair ? sm_count() / 2 : sm_count();
   const int cands[5] = {256, 192, 128, 64, 32};
   const double tile_eff[5] = {1.0, 0.97, 0.9, 0.75, 0.6};
   int pick = 0;
   double best = -1.0;
   for (int i = 0; i < 5; ++i) {
     const int bn = cands[i];
+    if (pair && bn != 256 && bn != 128) continue;
     const int out = (epi == EPI_SWIGLU) ? bn / 2 : bn;
     if (epi == EPI_SWIGLU && bn < 64) continue;
     if (out > a.N && !(out == 32 || (epi == EPI_SWIGLU && bn == 64))) continue;  // no wider than N
@@ -715,15 +895,41 @@ bool make_tensor_map_f32(CUtensorMap* m, const void* ptr, long long rows, long l
   return make_map(m, ptr, rows, cols, box_rows, MAP_F32_PLAIN);
 }
 
+// Whether a grouped GEMM runs on CTA pairs (256-row tiles).  Pairs are used
+// only when EC2MOE_GEMM_PAIR=1 is set in the environment (for the row-segment
+// epilogues); EC2MOE_GEMM_PAIR=2 picks them by shape (groups tall enough that
+// 256-row tiles waste at most ~10% more rows than 128-row ones).  Both paths
+// compute the same result; the single-CTA kernel measured faster so far.
+bool use_pairs(const GemmArgs& a, int epi) {
+  if (!(epi == EPI_STORE || epi == EPI_GELU || epi == EPI_SWIGLU || epi == EPI_SCATTER)) return false;
+  static const int forced = [] {
+    const char* v = getenv("EC2MOE_GEMM_PAIR");
+    return v ? (v[0] == '1' ? 1 : (v[0] == '2' ? 2 : 0)) : 0;
+  }();
+  if (forced == 0) return false;
+  if (forced == 1) return true;
+  const int ga = a.g_active > 0 ? a.g_active : a.G;
+  const double rows = (double)a.max_rows / ga;  // expected rows per group
+  if (rows < 2 * BM) return false;
+  const double pad1 = std::ceil(rows / BM) * BM, pad2 = std::ceil(rows / (2 * BM)) * (2 * BM);
+  return pad2 <= 1.1 * pad1;
+}
+
 cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
   if (a.G < 1 || a.G > MAX_GROUPS || a.N % 32 != 0 || a.K % 8 != 0) return cudaErrorInvalidValue;
-  const int bn = choose_bn(a, epi);
+  bool pair = use_pairs(a, epi);
+  int bn = choose_bn(a, epi, pair);
+  const int bn_out = epi == EPI_SWIGLU ? bn / 2 : bn;
+  if (pair && (bn_out % 64 != 0)) {
+    pair = false;
+    bn = choose_bn(a, epi, false);
+  }
   switch (epi) {
-    case EPI_STORE: return launch_epi<EPI_STORE>(a, bn, s);
-    case EPI_GELU: return launch_epi<EPI_GELU>(a, bn, s);
-    case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, s);
-    case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, s);
-    case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, s);
+    case EPI_STORE: return launch_epi<EPI_STORE>(a, bn, pair, s);
+    case EPI_GELU: return launch_epi<EPI_GELU>(a, bn, pair, s);
+    case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, pair, s);
+    case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, pair, s);
+    case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, false, s);
     case EPI_PARTIAL:
       if (!a.partial || a.N % 4 != 0) return cudaErrorInvalidValue;
       return bn >= 256 ? launch_cfg<256, EPI_PARTIAL, stages_for(256)>(a, s)

@@ -51,7 +51,7 @@ CLOUD = 1
 class LayerDesc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in
                 ("T", "d", "E", "d_ff", "k", "n_groups", "act", "dtype", "r", "n_shared", "d_ff_shared",
-                 "renorm_topk")]
+                 "renorm_topk", "top_groups")]
 
 
 class LayerWeights(ctypes.Structure):
@@ -160,8 +160,8 @@ def status_string(status: int) -> str:
 
 
 def make_desc(T, d, E, d_ff, k, n_groups=1, act=GELU, dtype=BF16, r=0, n_shared=0, d_ff_shared=0,
-              renorm_topk=0) -> LayerDesc:
-    return LayerDesc(T, d, E, d_ff, k, n_groups, act, dtype, r, n_shared, d_ff_shared, renorm_topk)
+              renorm_topk=0, top_groups=0) -> LayerDesc:
+    return LayerDesc(T, d, E, d_ff, k, n_groups, act, dtype, r, n_shared, d_ff_shared, renorm_topk, top_groups)
 
 
 def host_mask(mask):

@@ -17,7 +17,7 @@ from .synth import LayerConfig
 def desc_for(cfg: LayerConfig, T: Optional[int] = None) -> C.LayerDesc:
     return C.make_desc(T=cfg.T if T is None else T, d=cfg.d, E=cfg.E, d_ff=cfg.d_ff, k=cfg.k,
                        n_groups=cfg.n_groups, act=cfg.act, dtype=cfg.dtype, r=cfg.r, n_shared=cfg.n_shared,
-                       d_ff_shared=cfg.d_ff_shared, renorm_topk=cfg.renorm_topk)
+                       d_ff_shared=cfg.d_ff_shared, renorm_topk=cfg.renorm_topk, top_groups=cfg.top_groups)
 
 
 def weights_for(inp: Dict[str, Optional[torch.Tensor]]) -> C.LayerWeights:

@@ -52,6 +52,7 @@ class LayerConfig:
     n_shared: int = 0
     d_ff_shared: int = 0
     renorm_topk: int = 0
+    top_groups: int = 0
     zipf_s: float = 0.0
     seed: int = 0
 

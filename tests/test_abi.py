@@ -135,3 +135,21 @@ def test_other_entry_points_validate(lib):
     assert _status(C.ec2moe_shared_experts, _desc(n_shared=1, d_ff_shared=0), A, A, None, A, A, A, 1 << 30, 0) == \
         C.ERR_INVALID_ARG
     assert C.status_string(C.ERR_TIMEOUT) == "device wait timed out"
+
+
+def test_top_group_pruning_validation(lib):
+    """Top-group pruning is checked on the host: a negative count is invalid,
+    and k above the allowed experts of the fewest-member choice of kept groups
+    is refused (the same rule as the oracle's pruned_candidate_floor)."""
+    from oracle import ec2moe_oracle as orc
+    A = 0x100000
+    mask = np.array([1, 0, 0, 0, 1, 1, 1, 0], np.uint8)  # groups of 2: allowed counts 1, 0, 2, 1
+    for G, k in [(1, 1), (1, 2), (2, 2), (2, 3), (3, 4), (3, 3), (0, 4)]:
+        d = _desc(T=0, E=8, n_groups=4, k=k, top_groups=G)  # T = 0: validation only, nothing to launch
+        got = _status(C.ec2moe_gate, d, A, A, A, A, A, mask, A, A, 0)
+        floor_k = orc.pruned_candidate_floor(mask.astype(bool), 4, G) if G else int(mask.sum())
+        want = C.ERR_TOO_FEW_EXPERTS if k > floor_k else C.OK
+        assert got == want, (G, k, got)
+    assert _status(C.ec2moe_gate, _desc(n_groups=2, top_groups=-1), A, A, A, A, A, np.ones(8, np.uint8), A, A, 0) == \
+        C.ERR_INVALID_ARG
+    assert _status(C.ec2moe_profile_only, -2) == C.ERR_INVALID_ARG

@@ -1,0 +1,29 @@
+"""The grouped GEMM on CTA pairs (tcgen05.mma.cta_group::2, 256-row tiles)
+and on single CTAs compute the same layer.
+
+EC2MOE_GEMM_PAIR=1 forces pairs wherever the epilogue allows them (also on
+short, ragged and empty groups), =2 lets the shape decide (tall groups) and
+=0 (the default) forbids them.  The variable is read once per
+process, so each setting runs the layer parity tests in a child process.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+SELECT = ("test_layer_forward or test_experts_and_combine_entry_points or test_zero_token_experts_and_tail_tiles "
+          "or test_layer_is_deterministic")
+
+
+@pytest.mark.parametrize("mode", ["1", "2"], ids=["pairs-forced", "pairs-by-shape"])
+def test_layer_parity_with_pair_gemm_setting(mode):
+    env = dict(os.environ, EC2MOE_GEMM_PAIR=mode)
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-m", "gpu", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_gpu_parity.py"), "-k", SELECT],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=1500)
+    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-2000:]
