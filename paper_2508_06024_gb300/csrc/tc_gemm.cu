@@ -27,13 +27,14 @@
 // of A and its half of the B tile (for SwiGLU: the even CTA the W1 rows, the
 // odd one the W3 rows), so a CTA moves 2/3 of the operand bytes per k-block of
 // an unpaired 128 x 256 tile and the same shared memory holds 1.5x the stages.
-// The even CTA issues the MMAs; the odd CTA's MMA warp relays "stage s has
-// landed" from its own full barrier to the even CTA (remote mbarrier arrive),
-// so each CTA's copies complete on its own barriers and each can drain its own
-// copies after an abort.  MMA completion is committed to both CTAs' empty and
-// accumulator-full barriers (multicast); both CTAs' epilogue warps release an
-// accumulator on the even CTA's tmem_empty barrier.  TMEM is allocated for the
-// pair (cta_group::2), and a cluster barrier precedes its release.
+// The even CTA issues the MMAs.  Both CTAs' copies of a stage complete on the
+// even CTA's full barrier (the odd CTA's tensor copies name the peer barrier,
+// .cta_group::2), which the even CTA arms for the bytes of both.  MMA
+// completion is committed to both CTAs' empty and accumulator-full barriers
+// (multicast); both CTAs' epilogue warps release an accumulator on the even
+// CTA's tmem_empty barrier.  TMEM is allocated for the pair (cta_group::2), and
+// a cluster barrier precedes its release.  After an abort the odd CTA cannot
+// observe its own copies, so it waits a fixed, bounded time for them to land.
 //
 // Every mbarrier wait is bounded by a clock64 budget.  A wait that gives up
 // sets the device error word, raises a CTA-wide abort flag that ends every
@@ -125,8 +126,8 @@ struct Cfg {
   static constexpr int CW = 16;  // columns per TMEM load
   static_assert(PART % CW == 0, "epilogue chunks must tile each part exactly");
   static constexpr int TMEM_COLS = pow2_at_least(2 * BN);  // two accumulators
-  // mbarriers: full[S], empty[S], (PAIR) ready[S], tmem_full[2], tmem_empty[2], drain
-  static constexpr int N_BARS = (PAIR ? 3 : 2) * STAGES + 5;
+  // mbarriers: full[S], empty[S], tmem_full[2], tmem_empty[2], drain
+  static constexpr int N_BARS = 2 * STAGES + 5;
   static constexpr int STG_PITCH = CW * 2 + 16;          // bytes per staged row (padded)
   // Row-segment epilogue (contiguous or per-row destinations): the four warps
   // of a lane quadrant stage 32 rows x 64 columns (bf16, 128-byte rows,
@@ -166,8 +167,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::OFF_BARS);
   uint64_t* full = bars;
   uint64_t* empty = bars + STAGES;
-  uint64_t* ready = bars + 2 * STAGES;  // PAIR, even CTA: the odd CTA's stage s has landed
-  uint64_t* tfull = bars + (PAIR ? 3 : 2) * STAGES;
+  uint64_t* tfull = bars + 2 * STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tfull + 4;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_SLOT);
@@ -191,7 +191,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
       mbar_init(smem_u32(&empty[s]), 1);
-      if (PAIR) mbar_init(smem_u32(&ready[s]), 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
@@ -275,17 +274,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             break;
           }
           const uint32_t fb = smem_u32(&full[stage]);
-          mbar_expect_tx(fb, C::STAGE_BYTES);
-          tma_load_2d(smem_u32(sA + stage * C::A_BYTES), &tmA, kb * BK, a_row, fb);
-          if (EPI == EPI_SWIGLU && PAIR) {
-            // the even CTA stages the W1 rows of the tile, the odd CTA the W3 rows
-            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), rank ? &tmB2 : &tmB, kb * BK, b_row, fb);
-          } else if (EPI == EPI_SWIGLU) {
-            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK, b_row, fb);
-            tma_load_2d(smem_u32(sB + stage * C::B_BYTES + C::B_BYTES / 2), &tmB2, kb * BK, b_row, fb);
+          if (PAIR) {
+            // both halves complete on the even CTA's full barrier
+            if (rank == 0) mbar_expect_tx(fb, 2 * C::STAGE_BYTES);
+            const uint32_t fb0 = rank == 0 ? fb : map_to_rank(fb, 0);
+            tma_load_2d_to_pair_bar(smem_u32(sA + stage * C::A_BYTES), &tmA, kb * BK, a_row, fb0);
+            // SwiGLU: the even CTA stages the W1 rows of the tile, the odd CTA the W3 rows
+            const CUtensorMap* tb = (EPI == EPI_SWIGLU && rank) ? &tmB2 : &tmB;
+            tma_load_2d_to_pair_bar(smem_u32(sB + stage * C::B_BYTES), tb, kb * BK,
+                                    b_row + (EPI == EPI_SWIGLU ? 0 : static_cast<int>(rank) * C::CTA_B_ROWS), fb0);
           } else {
-            tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK,
-                        b_row + static_cast<int>(rank) * C::CTA_B_ROWS, fb);
+            mbar_expect_tx(fb, C::STAGE_BYTES);
+            tma_load_2d(smem_u32(sA + stage * C::A_BYTES), &tmA, kb * BK, a_row, fb);
+            if (EPI == EPI_SWIGLU) {
+              tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK, b_row, fb);
+              tma_load_2d(smem_u32(sB + stage * C::B_BYTES + C::B_BYTES / 2), &tmB2, kb * BK, b_row, fb);
+            } else {
+              tma_load_2d(smem_u32(sB + stage * C::B_BYTES), &tmB, kb * BK, b_row, fb);
+            }
           }
           issued |= 1u << stage;
           issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -297,35 +303,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       }
       if (!ok || *abort_flag) {
         // Let every copy this CTA started land before shared memory is released.
-        for (int s = 0; s < STAGES; ++s)
-          if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, DRAIN_CYCLES);
+        if (PAIR && rank != 0) {
+          // its copies complete on the even CTA's barriers: wait a fixed time
+          if (issued) {
+            const unsigned long long t0 = globaltimer_ns();
+            while (globaltimer_ns() - t0 < 200000ull) __nanosleep(1000);
+          }
+        } else {
+          for (int s = 0; s < STAGES; ++s)
+            if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, DRAIN_CYCLES);
+        }
       }
     }
   } else if (warp == 1) {
     if (PAIR && rank != 0) {
-      // ------------------------------------------------ odd CTA of a pair: relay
-      // Each stage of this CTA that has landed is announced to the even CTA,
-      // whose MMAs read it.
-      if (lane == 0) {
-        int stage = 0;
-        uint32_t phase = 0;
-        int cursor = 0;
-        bool ok = true;
-        for (int tile = tile_first; tile < n_tiles && ok; tile += tile_step) {
-          (void)decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
-          for (int kb = 0; kb < num_kb; ++kb) {
-            if (!mbar_wait(smem_u32(&full[stage]), phase, budget, abort_flag, &g_tc_error)) {
-              ok = false;
-              break;
-            }
-            mbar_arrive_remote(map_to_rank(smem_u32(&ready[stage]), 0));
-            if (++stage == STAGES) {
-              stage = 0;
-              phase ^= 1u;
-            }
-          }
-        }
-      }
+      // odd CTA of a pair: the even CTA issues the pair's MMAs
     } else if (lane == 0) {
       // ---------------------------------------------------------------- MMA issuer
       constexpr uint32_t IDESC = idesc_bf16(C::TILE_M, BN);
@@ -357,10 +349,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait(full0 + 8u * stage, phase, budget, abort_flag, &g_tc_error)) {
-            ok = false;
-            break;
-          }
-          if (PAIR && !mbar_wait_cluster(smem_u32(&ready[stage]), phase, budget, abort_flag, &g_tc_error)) {
             ok = false;
             break;
           }
@@ -895,16 +883,17 @@ bool make_tensor_map_f32(CUtensorMap* m, const void* ptr, long long rows, long l
   return make_map(m, ptr, rows, cols, box_rows, MAP_F32_PLAIN);
 }
 
-// Whether a grouped GEMM runs on CTA pairs (256-row tiles).  Pairs are used
-// only when EC2MOE_GEMM_PAIR=1 is set in the environment (for the row-segment
-// epilogues); EC2MOE_GEMM_PAIR=2 picks them by shape (groups tall enough that
-// 256-row tiles waste at most ~10% more rows than 128-row ones).  Both paths
-// compute the same result; the single-CTA kernel measured faster so far.
+// Whether a grouped GEMM runs on CTA pairs (256-row tiles): for the row-
+// segment epilogues, when the groups are tall enough that 256-row tiles waste
+// at most ~10% more rows than 128-row ones (the Mixtral-shaped and
+// fine-grained layers; the Switch-shaped one, with ~341 rows per expert, keeps
+// single CTAs).  EC2MOE_GEMM_PAIR=0 / =1 in the environment forbids / forces
+// pairs (A/B comparisons; both compute the same result).
 bool use_pairs(const GemmArgs& a, int epi) {
   if (!(epi == EPI_STORE || epi == EPI_GELU || epi == EPI_SWIGLU || epi == EPI_SCATTER)) return false;
   static const int forced = [] {
     const char* v = getenv("EC2MOE_GEMM_PAIR");
-    return v ? (v[0] == '1' ? 1 : (v[0] == '2' ? 2 : 0)) : 0;
+    return v ? (v[0] == '1' ? 1 : (v[0] == '0' ? 0 : 2)) : 2;
   }();
   if (forced == 0) return false;
   if (forced == 1) return true;

@@ -1,9 +1,9 @@
 """The grouped GEMM on CTA pairs (tcgen05.mma.cta_group::2, 256-row tiles)
 and on single CTAs compute the same layer.
 
-EC2MOE_GEMM_PAIR=1 forces pairs wherever the epilogue allows them (also on
-short, ragged and empty groups), =2 lets the shape decide (tall groups) and
-=0 (the default) forbids them.  The variable is read once per
+By default the shape decides (tall groups take pairs); EC2MOE_GEMM_PAIR=1
+forces pairs wherever the epilogue allows them (also on short, ragged and
+empty groups) and EC2MOE_GEMM_PAIR=0 forbids them.  The variable is read once per
 process, so each setting runs the layer parity tests in a child process.
 """
 import os
@@ -20,7 +20,7 @@ SELECT = ("test_layer_forward or test_experts_and_combine_entry_points or test_z
           "or test_layer_is_deterministic")
 
 
-@pytest.mark.parametrize("mode", ["1", "2"], ids=["pairs-forced", "pairs-by-shape"])
+@pytest.mark.parametrize("mode", ["1", "0"], ids=["pairs-forced", "pairs-off"])
 def test_layer_parity_with_pair_gemm_setting(mode):
     env = dict(os.environ, EC2MOE_GEMM_PAIR=mode)
     r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-m", "gpu", "-p", "no:cacheprovider",
