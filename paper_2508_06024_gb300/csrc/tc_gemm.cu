@@ -132,10 +132,11 @@ struct Cfg {
   // Row-segment epilogue (contiguous or per-row destinations): the four warps
   // of a lane quadrant stage 32 rows x 64 columns (bf16, 128-byte rows,
   // 16-byte chunks XOR-swizzled by row) and store whole 128-byte row
-  // segments.  EPI_REPLICATE keeps per-warp 32 x 16 chunks; EPI_PARTIAL
+  // segments (EPI_REPLICATE: to each of the row's destinations); EPI_PARTIAL
   // writes fp32 from registers.
-  static constexpr bool ROWSEG =
-      (EPI == EPI_STORE || EPI == EPI_GELU || EPI == EPI_SWIGLU || EPI == EPI_SCATTER) && BN_OUT % 64 == 0;
+  static constexpr bool ROWSEG = (EPI == EPI_STORE || EPI == EPI_GELU || EPI == EPI_SWIGLU || EPI == EPI_SCATTER ||
+                                  EPI == EPI_REPLICATE) &&
+                                 BN_OUT % 64 == 0;
   static constexpr int SLAB = 64;
   static constexpr int STG_BYTES =
       ROWSEG ? 4 * 32 * SLAB * 2 : (EPI == EPI_PARTIAL ? 0 : EPI_WARPS * 32 * STG_PITCH);
@@ -479,10 +480,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int pass = 0; pass < 2; ++pass) {
             const int rr = part * 8 + pass * 4 + (lane >> 3);
             const bool rvalid = __shfl_sync(0xffffffffu, valid ? 1 : 0, rr) != 0;
-            const long long drow = __shfl_sync(0xffffffffu, dest, rr);
             const U4 q4 = *reinterpret_cast<const U4*>(slab + rr * 128 + ((seg ^ (rr & 7)) * 16));
-            if (rvalid && col < p.N)
-              *reinterpret_cast<U4*>(reinterpret_cast<__nv_bfloat16*>(p.out) + drow * p.ldo + col) = q4;
+            __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(p.out);
+            if (EPI == EPI_REPLICATE) {
+              // the row's expert-order slots, then (optionally) its own row
+#pragma unroll
+              for (int r = 0; r < 8; ++r) {
+                if (r >= p.rep_k) break;  // uniform across the warp
+                const int dr = __shfl_sync(0xffffffffu, rdst[r], rr);
+                if (rvalid && col < p.N) *reinterpret_cast<U4*>(ob + (long long)dr * p.ldo + col) = q4;
+              }
+              const long long orow_r = __shfl_sync(0xffffffffu, out_row, rr);
+              if (rvalid && col < p.N && p.self_row_base >= 0)
+                *reinterpret_cast<U4*>(ob + (p.self_row_base + orow_r) * p.ldo + col) = q4;
+            } else {
+              const long long drow = __shfl_sync(0xffffffffu, dest, rr);
+              if (rvalid && col < p.N) *reinterpret_cast<U4*>(ob + drow * p.ldo + col) = q4;
+            }
           }
           asm volatile("bar.sync %0, 128;" ::"r"(1 + q) : "memory");
         }
@@ -822,7 +836,8 @@ constexpr int stages_for(int b_rows) {
 template <int EPI>
 cudaError_t launch_epi(const GemmArgs& a, int bn, bool pair, cudaStream_t s) {
   if (pair) {
-    if constexpr (EPI == EPI_STORE || EPI == EPI_GELU || EPI == EPI_SWIGLU || EPI == EPI_SCATTER) {
+    if constexpr (EPI == EPI_STORE || EPI == EPI_GELU || EPI == EPI_SWIGLU || EPI == EPI_SCATTER ||
+                  EPI == EPI_REPLICATE) {
       if (bn == 256) return launch_cfg<256, EPI, stages_for(128), true>(a, s);
       if (bn == 128) return launch_cfg<128, EPI, stages_for(64), true>(a, s);
     }
@@ -890,7 +905,8 @@ bool make_tensor_map_f32(CUtensorMap* m, const void* ptr, long long rows, long l
 // single CTAs).  EC2MOE_GEMM_PAIR=0 / =1 in the environment forbids / forces
 // pairs (A/B comparisons; both compute the same result).
 bool use_pairs(const GemmArgs& a, int epi) {
-  if (!(epi == EPI_STORE || epi == EPI_GELU || epi == EPI_SWIGLU || epi == EPI_SCATTER)) return false;
+  if (!(epi == EPI_STORE || epi == EPI_GELU || epi == EPI_SWIGLU || epi == EPI_SCATTER || epi == EPI_REPLICATE))
+    return false;
   static const int forced = [] {
     const char* v = getenv("EC2MOE_GEMM_PAIR");
     return v ? (v[0] == '1' ? 1 : (v[0] == '0' ? 0 : 2)) : 2;
@@ -918,7 +934,7 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
     case EPI_GELU: return launch_epi<EPI_GELU>(a, bn, pair, s);
     case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, pair, s);
     case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, pair, s);
-    case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, false, s);
+    case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, pair, s);
     case EPI_PARTIAL:
       if (!a.partial || a.N % 4 != 0) return cudaErrorInvalidValue;
       return bn >= 256 ? launch_cfg<256, EPI_PARTIAL, stages_for(256)>(a, s)
