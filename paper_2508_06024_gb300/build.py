@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libec2moe.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "gate.cu", "gate_tc.cu", "route.cu", "tc_gemm.cu", "simt_gemm.cu", "codec.cu", "skinny.cu", "sched.cpp"]
+SOURCES = ["api.cu", "gate.cu", "gate_tc.cu", "route.cu", "tc_gemm.cu", "simt_gemm.cu", "codec.cu", "skinny.cu", "tc_swap.cu", "sched.cpp"]
 
 
 def nvcc() -> str:

@@ -231,14 +231,19 @@ ec2moe_status check_mask(const ec2moe_layer_desc* d, const uint8_t* mask, uint32
 constexpr int SPLITK_MAX = 8;
 bool splitk_possible(const ec2moe_layer_desc* d) {
   const long long n = (long long)d->T * d->k;
-  return d->dtype == EC2MOE_BF16 && n > 4 && n <= 128 && d->d_ff >= 4096 && d->d % 4 == 0;
+  return d->dtype == EC2MOE_BF16 && n >= 1 && n <= 128 && d->d_ff >= 4096 && d->d % 4 == 0;
 }
-// The split whose (tile x K range) units fill whole waves of the SMs best
-// (expected m-tiles: one per expert with rows, at least n / 128).
+// The split whose (tile x K range) units fill whole waves of the SMs best.
+// Groups of at most SWAP_MAX_ROWS rows go to the swapped tensor-core kernel
+// (d / 128 weight tiles per expert with rows); otherwise the expected m-tiles
+// are one per expert with rows, at least n / 128, with d / 256 tiles each.
 int splitk_factor(const ec2moe_layer_desc* d, int n_allowed) {
   if (!splitk_possible(d)) return 1;
   const long long n = (long long)d->T * d->k;
   const long long experts = n < n_allowed ? n : n_allowed;
+  if (swap_gemm_enabled() && n <= SWAP_MAX_ROWS)
+    return swap_split_factor(experts * swap_tiles_per_group(d->d, EPI_PARTIAL), d->d_ff, SPLITK_MAX);
+  if (n <= 4) return 1;  // the weight-streaming kernel takes the whole K
   const long long m_tiles = experts > (n + 127) / 128 ? experts : (n + 127) / 128;
   const long long tiles = m_tiles * ((d->d + 255) / 256);
   const long long sms = sm_count();
@@ -315,7 +320,9 @@ GemmArgs gemm_base() {
 
 cudaError_t run_gemm(const ec2moe_layer_desc* d, const GemmArgs& g, int epi, cudaStream_t s) {
   if (!is_bf16(d)) return launch_gemm_simt(g, epi, s);
-  // decode-sized groups: stream each weight row once on the CUDA cores
+  // decode-sized groups: weight rows on the MMA's M side (tensor cores), else
+  // streamed once on the CUDA cores
+  if (gemm_swap_supported(g, epi)) return launch_gemm_swap(g, epi, s);
   if (gemm_skinny_supported(g, epi)) return launch_gemm_skinny(g, epi, s);
   return launch_gemm_tc(g, epi, s);
 }
@@ -989,12 +996,13 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
 
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream) {
   if (cudaStreamSynchronize(stream) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  unsigned int word = 0, word2 = 0, word3 = 0, word4 = 0;
+  unsigned int word = 0, word2 = 0, word3 = 0, word4 = 0, word5 = 0;
   if (read_tc_error(&word) != cudaSuccess) return EC2MOE_ERR_CUDA;
   if (read_codec_error(&word2) != cudaSuccess) return EC2MOE_ERR_CUDA;
   if (read_gate_error(&word3) != cudaSuccess) return EC2MOE_ERR_CUDA;
   if (read_route_error(&word4) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  if (word | word2 | word3) return EC2MOE_ERR_TIMEOUT;
+  if (read_swap_error(&word5) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (word | word2 | word3 | word5) return EC2MOE_ERR_TIMEOUT;
   return word4 ? EC2MOE_ERR_INVALID_ARG : EC2MOE_OK;
 }
 

@@ -180,6 +180,21 @@ cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s);  // fp
 // on the CUDA cores; every epilogue but EPI_REPLICATE.
 bool gemm_skinny_supported(const GemmArgs& a, int epi);
 cudaError_t launch_gemm_skinny(const GemmArgs& a, int epi, cudaStream_t s);
+// bf16 groups of at most SWAP_MAX_ROWS rows on the tensor cores with the
+// operands swapped (weight rows on the MMA's M side, tokens on N = 16);
+// every epilogue but EPI_REPLICATE.  EPI_PARTIAL needs a split_k that leaves
+// no K range of 64-column blocks empty (swap_split_factor picks one).
+constexpr int SWAP_MAX_ROWS = 16;
+bool swap_gemm_enabled();  // false when EC2MOE_GEMM_SWAP=0 is set in the environment
+bool gemm_swap_supported(const GemmArgs& a, int epi);
+cudaError_t launch_gemm_swap(const GemmArgs& a, int epi, cudaStream_t s);
+// Weight tiles of one group along N for the swapped kernel.
+long long swap_tiles_per_group(int N, int epi);
+// The K-range count (<= max_split, no empty range) whose `tiles` x ranges
+// units fill whole waves of one CTA per SM best.
+int swap_split_factor(long long tiles, int K, int max_split);
+// Reads and clears the swapped kernel's device error word (synchronous).
+cudaError_t read_swap_error(unsigned int* word);
 // 2-D bf16 tensor map over a row-major [rows, cols] matrix: box 64 columns x
 // box_rows rows, 128-byte swizzle, zero fill out of bounds (cached).
 bool make_tensor_map_bf16(CUtensorMap* m, const void* ptr, long long rows, long long cols, int box_rows);

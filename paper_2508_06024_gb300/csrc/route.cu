@@ -508,7 +508,11 @@ cudaError_t launch_splitk_sum(const float* partial, int S, long long rows, int N
 // Split-K expert outputs (bf16 layers): for every token and 8-column chunk,
 // the k slots' fp32 partial sums over the K ranges are added (range order),
 // weighted by the slot's gate weight (slot order), plus the shared experts'
-// rows; one bf16 rounding at the end.
+// rows; one bf16 rounding at the end.  A decode step has only T * d / 8
+// threads, so latency decides: every slot's row position is read first, and
+// the S <= COMBINE_MAX_S range loads of a slot are issued together.
+constexpr int COMBINE_MAX_S = 8;
+constexpr int COMBINE_MAX_K = 8;
 __global__ void splitk_combine_kernel(const float* __restrict__ partial, int S, long long part_rows,
                                       const int32_t* __restrict__ offsets, const int32_t* __restrict__ idx,
                                       const int32_t* __restrict__ rel, int rel_mode, const float* __restrict__ w,
@@ -525,21 +529,36 @@ __global__ void splitk_combine_kernel(const float* __restrict__ partial, int S, 
     float acc[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) acc[j] = 0.0f;
-    for (int slot = 0; slot < k; ++slot) {
-      const long long entry = t * k + slot;
-      const long long pos = rel_mode ? (long long)offsets[idx[entry]] + rel[entry] : (long long)rel[entry];
+    long long pos[COMBINE_MAX_K];
+    float wt[COMBINE_MAX_K];
+#pragma unroll
+    for (int slot = 0; slot < COMBINE_MAX_K; ++slot) {
+      pos[slot] = 0;
+      wt[slot] = 0.0f;
+      if (slot < k) {
+        const long long entry = t * k + slot;
+        pos[slot] = rel_mode ? (long long)offsets[idx[entry]] + rel[entry] : (long long)rel[entry];
+        wt[slot] = w[entry];
+      }
+    }
+#pragma unroll
+    for (int slot = 0; slot < COMBINE_MAX_K; ++slot) {
+      if (slot >= k) break;
+      float v[COMBINE_MAX_S][8];
+#pragma unroll
+      for (int s = 0; s < COMBINE_MAX_S; ++s)
+        if (s < S) load8(partial + ((long long)s * part_rows + pos[slot]) * d + c, v[s]);
       float sum[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) sum[j] = 0.0f;
-      for (int s = 0; s < S; ++s) {
-        float v[8];
-        load8(partial + ((long long)s * part_rows + pos) * d + c, v);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) sum[j] += v[j];
-      }
-      const float wt = w[entry];
+      for (int s = 0; s < COMBINE_MAX_S; ++s)
+        if (s < S) {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) acc[j] = fmaf(wt, sum[j], acc[j]);
+          for (int j = 0; j < 8; ++j) sum[j] += v[s][j];
+        }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) acc[j] = fmaf(wt[slot], sum[j], acc[j]);
     }
     for (int j = 0; j < n_shared; ++j) {
       float v[8];
@@ -555,6 +574,7 @@ cudaError_t launch_splitk_combine(const float* partial, int split_k, long long p
                                   const int32_t* idx, const int32_t* rel, bool rel_mode, const float* w,
                                   const void* shared, int n_shared, void* Y, int T, int k, int d, cudaStream_t s) {
   if (T <= 0) return cudaSuccess;
+  if (split_k < 1 || split_k > COMBINE_MAX_S || k < 1 || k > COMBINE_MAX_K) return cudaErrorInvalidValue;
   const long long total = (long long)T * (d / 8);
   long long blocks = (total + 255) / 256;
   const long long cap = (long long)sm_count() * 8;

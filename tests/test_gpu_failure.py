@@ -28,8 +28,10 @@ def lib():
 @pytest.mark.parametrize("cfg", [S.preset("switch_bf16", T=512, seed=31),
                                  S.preset("finegrained_bf16", T=300, seed=32),
                                  # ~2730 rows per expert: the expert GEMMs run on CTA pairs
-                                 S.preset("mixtral_bf16", T=4096, E=4, n_allowed=3, d_ff=1024, seed=33)],
-                         ids=["switch", "finegrained", "mixtral-pairs"])
+                                 S.preset("mixtral_bf16", T=4096, E=4, n_allowed=3, d_ff=1024, seed=33),
+                                 # two rows: expert GEMMs with the operands swapped, split-K down projection
+                                 S.preset("decode_bf16", T=1, d_ff=4096, seed=34)],
+                         ids=["switch", "finegrained", "mixtral-pairs", "decode-swap"])
 def test_zero_wait_budget_times_out_and_recovers(cfg):
     inp = S.make_inputs(cfg, device="cuda")
     run = LayerRun(cfg, inp)
