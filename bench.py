@@ -182,14 +182,22 @@ def roofline_for(cfg, name, avg_ms, peaks, peaks_src, traffic, touched: int = 0)
 
 
 def committed_traffic(cfg, kernel):
-    """dram read+write bytes per launch for (workload, kernel) from profiles/traffic.txt, or None."""
+    """dram read+write bytes per launch for (workload, kernel) from profiles/traffic.txt, or None.
+
+    A row keyed ``name@T=n`` holds for that token count; a row keyed by the
+    bare preset name holds for the preset's own token count only."""
+    from paper_2508_06024_gb300 import synth as S
+
     p = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(p):
         return None
+    keys = {f"{cfg.name}@T={cfg.T}"}
+    if cfg.T == S.preset(cfg.name).T:
+        keys.add(cfg.name)
     with open(p) as f:
         for line in f:
             parts = line.split()
-            if len(parts) >= 3 and not line.startswith("#") and parts[0] == cfg.name and parts[1] == kernel:
+            if len(parts) >= 3 and not line.startswith("#") and parts[0] in keys and parts[1] == kernel:
                 return float(parts[2])
     return None
 

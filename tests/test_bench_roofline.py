@@ -51,3 +51,8 @@ def test_committed_traffic_lookup():
     up = bench.committed_traffic(sw, "expert_up")
     assert up is not None and 0.5 < up / bench.kernel_work(sw, "expert_up")[1] < 1.5
     assert bench.committed_traffic(sw, "no_such_kernel") is None
+    # a bare preset name holds for the preset's own token count only
+    assert bench.committed_traffic(sw.replace(T=2048), "expert_up") is None
+    dec = S.preset("decode_bf16", T=1)
+    assert bench.committed_traffic(dec, "expert_up") is not None
+    assert bench.committed_traffic(S.preset("decode_bf16", T=2), "expert_up") is None
