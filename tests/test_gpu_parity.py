@@ -218,6 +218,10 @@ LAYER_CASES = [
     (S.preset("switch_bf16", T=2, seed=43), None),
     (S.preset("decode_bf16", T=1, n_allowed=8, r=256, seed=46), None),
     (S.preset("mixtral_bf16", T=3, seed=44), None),
+    # split-K reduce inside the swapped-operand down projection: all 16 entries
+    # (T = 8, Top-2) and Top-3 with relative row placement
+    (S.preset("decode_bf16", T=8, n_allowed=8, r=256, seed=61), None),
+    (S.preset("decode_bf16", T=5, k=3, n_allowed=6, r=128, seed=62), None),
     # split-K encoder with a K range count the k-block count does not divide
     # (33 k-blocks of 64 in 11 ranges of 3)
     (S.preset("decode_bf16", T=7, d=2112, d_ff=2048, n_allowed=8, r=256, seed=49), None),
