@@ -215,9 +215,13 @@ __device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
   return r;
 }
-// Arrive (release, cluster scope) on an mbarrier of another CTA of the cluster.
+// Arrive on an mbarrier of another CTA of the cluster, with the default
+// semantics (release at CTA scope).  The epilogue's release of a TMEM
+// accumulator orders only its tcgen05.ld (through tcgen05.fence), not its
+// global stores, so a cluster-scope release -- which waits until every prior
+// store of the thread is acknowledged -- is not needed.
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
   uint32_t ok;
