@@ -253,30 +253,60 @@ __global__ void gather_rel_kernel(const uint8_t* __restrict__ src, uint8_t* __re
   }
 }
 
-// y[t] = sum_s slot[t*k+s] + sum_j shared[j*T+t] in that order, fp32 sum.
+// Eight consecutive elements held as loaded (bf16: 16 bytes, fp32: 32 bytes).
 template <typename TE>
+struct Raw8;
+template <>
+struct Raw8<__nv_bfloat16> {
+  U4 q;
+  __device__ __forceinline__ void load(const __nv_bfloat16* p) { q = *reinterpret_cast<const U4*>(p); }
+  __device__ __forceinline__ void add_to(float* acc) const {
+    acc[0] += bf16_lo(q.x); acc[1] += bf16_hi(q.x); acc[2] += bf16_lo(q.y); acc[3] += bf16_hi(q.y);
+    acc[4] += bf16_lo(q.z); acc[5] += bf16_hi(q.z); acc[6] += bf16_lo(q.w); acc[7] += bf16_hi(q.w);
+  }
+};
+template <>
+struct Raw8<float> {
+  float4 a, b;
+  __device__ __forceinline__ void load(const float* p) {
+    a = *reinterpret_cast<const float4*>(p);
+    b = *reinterpret_cast<const float4*>(p + 4);
+  }
+  __device__ __forceinline__ void add_to(float* acc) const {
+    acc[0] += a.x; acc[1] += a.y; acc[2] += a.z; acc[3] += a.w;
+    acc[4] += b.x; acc[5] += b.y; acc[6] += b.z; acc[7] += b.w;
+  }
+};
+constexpr int CB_MAX_K = 8;       // Top-k limit of the ABI
+constexpr int CB_MAX_SHARED = 4;  // shared-expert limit of the ABI
+static_assert(CB_MAX_K == EC2MOE_MAX_TOPK && CB_MAX_SHARED == EC2MOE_MAX_SHARED, "combine limits follow the ABI");
+
+// y[t] = sum_s slot[t*k+s] + sum_j shared[j*T+t] in that order, fp32 sum.
+// All k + n_shared <= R rows of an 8-column chunk are loaded before the first
+// add, so a thread keeps them in flight together; R is the smallest of 2, 4,
+// 8, 12 that holds them, so the register count (and occupancy) follows the
+// rows a token actually has.
+template <typename TE, int R>
 __global__ void combine_kernel(const TE* __restrict__ slot, const TE* __restrict__ shared, int n_shared,
                                TE* __restrict__ Y, int T, int k, int d) {
   pdl_trigger();
   pdl_wait();
   const int per_row = d / 8;
+  const int rows = k + n_shared;
   const long long total = (long long)T * per_row;
   for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
        i += (long long)gridDim.x * blockDim.x) {
     const long long t = i / per_row;
     const int c = static_cast<int>(i % per_row) * 8;
+    Raw8<TE> r[R];
+#pragma unroll
+    for (int q = 0; q < R; ++q)
+      if (q < rows)
+        r[q].load(q < k ? slot + (t * k + q) * d + c : shared + ((long long)(q - k) * T + t) * d + c);
     float acc[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-    float v[8];
-    for (int s = 0; s < k; ++s) {
-      load8(slot + (t * k + s) * d + c, v);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) acc[j] += v[j];
-    }
-    for (int j = 0; j < n_shared; ++j) {
-      load8(shared + ((long long)j * T + t) * d + c, v);
-#pragma unroll
-      for (int q = 0; q < 8; ++q) acc[q] += v[q];
-    }
+    for (int q = 0; q < R; ++q)
+      if (q < rows) r[q].add_to(acc);
     store8(Y + t * d + c, acc);
   }
 }
@@ -591,22 +621,35 @@ cudaError_t launch_splitk_combine(const float* partial, int split_k, long long p
 cudaError_t launch_combine(const void* slot, const void* shared, int n_shared, void* Y, int T, int k, int d, bool bf16,
                            cudaStream_t s) {
   if (T <= 0) return cudaSuccess;
+  if (k < 1 || k > CB_MAX_K || n_shared < 0 || n_shared > CB_MAX_SHARED) return cudaErrorInvalidValue;
   const long long total = (long long)T * (d / 8);
   long long blocks = (total + 255) / 256;
   const long long cap = (long long)sm_count() * 8;
   if (blocks > cap) blocks = cap;
   KernelScope ks("combine", s);
+  const int ns = shared ? n_shared : 0;
+  const int rows = k + ns;
+  cudaError_t e;
   if (bf16) {
-    cudaError_t e = launch_kernel(combine_kernel<__nv_bfloat16>, dim3(static_cast<int>(blocks)), dim3(256), 0, s,
-                                  static_cast<const __nv_bfloat16*>(slot), static_cast<const __nv_bfloat16*>(shared),
-                                  shared ? n_shared : 0, static_cast<__nv_bfloat16*>(Y), T, k, d);
-    if (e != cudaSuccess) return e;
+    const auto* sl = static_cast<const __nv_bfloat16*>(slot);
+    const auto* sh = static_cast<const __nv_bfloat16*>(shared);
+    auto* y = static_cast<__nv_bfloat16*>(Y);
+    const dim3 g(static_cast<int>(blocks));
+    if (rows <= 2) e = launch_kernel(combine_kernel<__nv_bfloat16, 2>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
+    else if (rows <= 4) e = launch_kernel(combine_kernel<__nv_bfloat16, 4>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
+    else if (rows <= 8) e = launch_kernel(combine_kernel<__nv_bfloat16, 8>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
+    else e = launch_kernel(combine_kernel<__nv_bfloat16, 12>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
   } else {
-    cudaError_t e = launch_kernel(combine_kernel<float>, dim3(static_cast<int>(blocks)), dim3(256), 0, s,
-                                  static_cast<const float*>(slot), static_cast<const float*>(shared),
-                                  shared ? n_shared : 0, static_cast<float*>(Y), T, k, d);
-    if (e != cudaSuccess) return e;
+    const auto* sl = static_cast<const float*>(slot);
+    const auto* sh = static_cast<const float*>(shared);
+    auto* y = static_cast<float*>(Y);
+    const dim3 g(static_cast<int>(blocks));
+    if (rows <= 2) e = launch_kernel(combine_kernel<float, 2>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
+    else if (rows <= 4) e = launch_kernel(combine_kernel<float, 4>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
+    else if (rows <= 8) e = launch_kernel(combine_kernel<float, 8>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
+    else e = launch_kernel(combine_kernel<float, 12>, g, dim3(256), 0, s, sl, sh, ns, y, T, k, d);
   }
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
