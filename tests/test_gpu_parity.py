@@ -229,6 +229,7 @@ LAYER_CASES = [
     # with several token tiles, 72 gate rows, and an fp32 layer
     (S.preset("mixtral_bf16", T=129, seed=50), None),
     (S.preset("finegrained_bf16", T=200, seed=51), None),
+    (S.preset("finegrained_bf16", T=150, seed=63), None),
     (S.preset("tiny_fp32", T=100, d=1024, seed=52), None),
     (S.preset("tiny_fp32", T=7, seed=45), None),
     # the limits: 128 experts in 16 groups, Top-8, 144 gate rows; and many
