@@ -222,7 +222,11 @@ ec2moe_status ec2moe_route_noalloc(const ec2moe_layer_desc* desc, const int32_t*
  *  topk_w    fp32 [T, k] (ec2moe_gate)
  *  slot_out  out [T * k, d]: slot_out[t * k + s] = topk_w[t, s] * E_e(x_t)
  *            for e = topk_idx[t, s]
- *  workspace ec2moe_experts_workspace_size bytes */
+ *  workspace ec2moe_experts_workspace_size bytes
+ * offsets and perm are read on the device: a group whose range is not inside
+ * [0, T * k] (or is decreasing) and a perm entry outside [0, T * k) are
+ * skipped, with nothing written for them, and ec2moe_last_device_error then
+ * reports EC2MOE_ERR_INVALID_ARG. */
 ec2moe_status ec2moe_experts(const ec2moe_layer_desc* desc, const void* X_perm, const int32_t* offsets,
                              const void* W1, const void* W3, const void* W2, const float* topk_w,
                              const int32_t* perm, void* slot_out, void* workspace, size_t ws_bytes,
@@ -271,10 +275,12 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
                                    size_t ws_bytes, ec2moe_stream_t stream);
 
 /* Synchronises `stream`, then reads and clears the device error words of the
- * current device: EC2MOE_OK, EC2MOE_ERR_TIMEOUT when a bounded wait in a
- * tensor-core kernel gave up, EC2MOE_ERR_INVALID_ARG when a routing kernel met
- * (and skipped) an expert id outside [0, E) in a caller's topk_idx, or
- * EC2MOE_ERR_CUDA when the stream reports an error. */
+ * current device: EC2MOE_OK; EC2MOE_ERR_TIMEOUT when a bounded wait in a
+ * tensor-core kernel gave up; EC2MOE_ERR_INVALID_ARG when a routing kernel met
+ * (and skipped) an expert id outside [0, E) in a caller's topk_idx, or a
+ * grouped expert GEMM met (and skipped) a group range in `offsets` outside
+ * [0, T * k] or a destination in `perm` outside [0, T * k); EC2MOE_ERR_CUDA
+ * when the stream reports an error.  A timeout takes precedence. */
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream);
 
 /* Budget, in SM clock cycles, of every bounded wait inside the tensor-core

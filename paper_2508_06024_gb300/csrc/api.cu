@@ -996,14 +996,20 @@ ec2moe_status ec2moe_layer_forward_pipelined(const ec2moe_layer_desc* desc, cons
 
 ec2moe_status ec2moe_last_device_error(ec2moe_stream_t stream) {
   if (cudaStreamSynchronize(stream) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  unsigned int word = 0, word2 = 0, word3 = 0, word4 = 0, word5 = 0;
-  if (read_tc_error(&word) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  if (read_codec_error(&word2) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  if (read_gate_error(&word3) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  if (read_route_error(&word4) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  if (read_swap_error(&word5) != cudaSuccess) return EC2MOE_ERR_CUDA;
-  if (word | word2 | word3 | word5) return EC2MOE_ERR_TIMEOUT;
-  return word4 ? EC2MOE_ERR_INVALID_ARG : EC2MOE_OK;
+  unsigned int tc = 0, codec = 0, gate = 0, route = 0, swap = 0, skinny = 0, simt = 0;
+  if (read_tc_error(&tc) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (read_codec_error(&codec) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (read_gate_error(&gate) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (read_route_error(&route) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (read_swap_error(&swap) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (read_skinny_error(&skinny) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  if (read_simt_error(&simt) != cudaSuccess) return EC2MOE_ERR_CUDA;
+  // bit 0 of the GEMM, codec and gate words: a bounded wait timed out;
+  // bit 1 of the GEMM words and any bit of the routing word: an index outside
+  // the call's rows or experts was skipped
+  if ((tc | codec | gate | swap) & 1u) return EC2MOE_ERR_TIMEOUT;
+  if (((tc | swap | skinny | simt) & 2u) || route) return EC2MOE_ERR_INVALID_ARG;
+  return EC2MOE_OK;
 }
 
 int32_t ec2moe_last_launch_count(void) { return launch_count(); }

@@ -228,7 +228,12 @@ cudaError_t read_codec_error(unsigned int* word);
 cudaError_t read_gate_error(unsigned int* word);
 
 // Reads and clears the tensor-core kernels' device error word (synchronous).
+// In the grouped-GEMM words (tensor-core, swapped, weight-streaming, SIMT)
+// bit 0 is a timed-out wait and bit 1 a group range (offsets) or a scatter
+// destination (perm) outside the call's rows, skipped.
 cudaError_t read_tc_error(unsigned int* word);
+cudaError_t read_skinny_error(unsigned int* word);
+cudaError_t read_simt_error(unsigned int* word);
 // Reads and clears the routing kernels' device error word (synchronous):
 // nonzero when an expert id outside [0, E) or a permutation entry outside
 // [0, rows) was met (and skipped).

@@ -14,6 +14,10 @@
 #include "internal.h"
 
 namespace ec2moe {
+// bit 1: a group range (offsets) or a scatter destination (perm) outside the
+// rows of the call was skipped
+__device__ unsigned int g_simt_error;
+
 namespace {
 
 constexpr int TM = 64, TN = 64, TK = 16;
@@ -35,6 +39,7 @@ struct SParams {
   long long self_row_base;
   int n_tiles_n;
   long long a_rows, b_rows;
+  long long row_limit;  // rows of the call: group ranges and scatter destinations lie in [0, row_limit)
 };
 
 template <int EPI>
@@ -54,6 +59,12 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SParams p) {
       if (p.offsets) {
         r0 = p.offsets[g];
         mg = p.offsets[g + 1] - r0;
+        if (r0 < 0 || mg < 0 || static_cast<long long>(r0) + mg > p.row_limit) {
+          // not a range of this call's rows: the group is skipped
+          atomicOr(&g_simt_error, 2u);
+          r0 = 0;
+          mg = 0;
+        }
       } else {
         r0 = g * p.M;
         mg = p.M;
@@ -117,6 +128,10 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(const SParams p) {
       float sc = 1.0f;
       if (EPI == EPI_SCATTER) {
         dest = p.perm ? p.perm[out_row] : out_row;
+        if (dest < 0 || dest >= p.row_limit) {
+          atomicOr(&g_simt_error, 2u);
+          continue;
+        }
         if (p.scale) sc = p.scale[dest];
       }
 #pragma unroll
@@ -147,6 +162,7 @@ cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s) {
   p.B = static_cast<const float*>(a.B);
   p.B2 = static_cast<const float*>(a.B2);
   p.offsets = a.offsets;
+  p.row_limit = a.max_rows > 0 ? a.max_rows : (1LL << 62);
   p.G = a.G;
   p.M = a.M;
   p.a_shared = a.a_shared;
@@ -179,6 +195,13 @@ cudaError_t launch_gemm_simt(const GemmArgs& a, int epi, cudaStream_t s) {
   }
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+cudaError_t read_simt_error(unsigned int* word) {
+  unsigned int zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(word, g_simt_error, sizeof(unsigned int));
+  if (e != cudaSuccess) return e;
+  return cudaMemcpyToSymbol(g_simt_error, &zero, sizeof(unsigned int));
 }
 
 }  // namespace ec2moe

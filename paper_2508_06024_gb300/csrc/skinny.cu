@@ -19,6 +19,11 @@
 #include "internal.h"
 
 namespace ec2moe {
+
+// bit 1: a group range (offsets) or a scatter destination (perm) outside the
+// rows of the call was skipped
+__device__ unsigned int g_skinny_error;
+
 namespace {
 
 constexpr int SK_WARPS = 8;
@@ -39,6 +44,7 @@ struct SkParams {
   const int32_t* perm;
   const float* scale;
   int n_blocks;  // column blocks per group
+  long long row_limit;  // rows of the call: group ranges and scatter destinations lie in [0, row_limit)
 };
 
 __device__ __forceinline__ void dot8(const U4& w, const float* a, float& acc) {
@@ -65,6 +71,11 @@ __device__ __forceinline__ SkUnit next_unit(const SkParams& p, int u, int units)
     if (p.offsets) {
       r0 = p.offsets[g];
       mg = p.offsets[g + 1] - r0;
+      if (r0 < 0 || mg < 0 || static_cast<long long>(r0) + mg > p.row_limit) {
+        // not a range of this call's rows: the group is skipped
+        atomicOr(&g_skinny_error, 2u);
+        mg = 0;
+      }
     } else {
       r0 = g * p.M;
       mg = p.M;
@@ -205,11 +216,14 @@ __global__ void __launch_bounds__(SK_THREADS) skinny_kernel(const SkParams p) {
           if (EPI == EPI_SWIGLU) y = silu_bf16out(v) * v2;
           else if (EPI == EPI_GELU) y = gelu_bf16out(v);
           else y = v;
+          bool ok = true;
           if (EPI == EPI_SCATTER) {
             dest = p.perm ? p.perm[out_row] : out_row;
-            if (p.scale) y *= p.scale[dest];
+            ok = dest >= 0 && dest < p.row_limit;
+            if (!ok) atomicOr(&g_skinny_error, 2u);
+            else if (p.scale) y *= p.scale[dest];
           }
-          p.out[dest * p.ldo + n0 + cc] = __float2bfloat16_rn(y);
+          if (ok) p.out[dest * p.ldo + n0 + cc] = __float2bfloat16_rn(y);
         }
       }
     if (nxt.u >= units) break;
@@ -268,6 +282,7 @@ cudaError_t launch_gemm_skinny(const GemmArgs& a, int epi, cudaStream_t s) {
   p.perm = a.perm;
   p.scale = a.scale;
   p.n_blocks = (a.N + SK_WARPS * SK_CPW - 1) / (SK_WARPS * SK_CPW);
+  p.row_limit = a.max_rows > 0 ? a.max_rows : (1LL << 62);
   const long long units = (long long)a.G * p.n_blocks;
   const long long cap = (long long)sm_count() * 8;
   const int grid = (int)(units < cap ? units : cap);
@@ -278,6 +293,13 @@ cudaError_t launch_gemm_skinny(const GemmArgs& a, int epi, cudaStream_t s) {
                                      : (rb <= 8 ? launch_r<8>(p, epi, grid, s) : launch_r<16>(p, epi, grid, s)));
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+cudaError_t read_skinny_error(unsigned int* word) {
+  unsigned int zero = 0;
+  cudaError_t e = cudaMemcpyFromSymbol(word, g_skinny_error, sizeof(unsigned int));
+  if (e != cudaSuccess) return e;
+  return cudaMemcpyToSymbol(g_skinny_error, &zero, sizeof(unsigned int));
 }
 
 }  // namespace ec2moe

@@ -59,7 +59,9 @@
 
 namespace ec2moe {
 
-__device__ unsigned int g_tc_error;  // bit 0: a bounded wait timed out
+// bit 0: a bounded wait timed out; bit 1: a group range (offsets) or a
+// scatter destination (perm) outside the rows of the call was skipped
+__device__ unsigned int g_tc_error;
 
 namespace {
 
@@ -93,6 +95,7 @@ struct Params {
   int split_k, kb_per_split;
   float* partial;
   long long part_rows;
+  long long row_limit;  // rows of the call: group ranges and scatter destinations lie in [0, row_limit)
 };
 
 // ------------------------------------------------------------------ tile schedule
@@ -212,6 +215,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (p.offsets) {
             r0 = p.offsets[g];
             mg = p.offsets[g + 1] - r0;
+            if (r0 < 0 || mg < 0 || static_cast<long long>(r0) + mg > p.row_limit) {
+              // not a range of this call's rows: the group is skipped
+              atomicOr(&g_tc_error, 2u);
+              r0 = 0;
+              mg = 0;
+            }
           }
           row0[g] = r0;
           return (mg + C::TILE_M - 1) / C::TILE_M;
@@ -402,15 +411,22 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       const int acc = it & 1;
       const uint32_t acc_phase = (it >> 1) & 1;
       // Row metadata first: its global loads overlap the tile's main loop.
+      // (a group's tiles exist only if the prologue accepted its range)
       const int mg = p.offsets ? (p.offsets[tc.g + 1] - p.offsets[tc.g]) : p.M;
       const int local = tc.m_blk * C::TILE_M + static_cast<int>(rank) * BM + row_in_tile;
-      const bool valid = local < mg;
+      bool valid = local < mg;
       const long long out_row = p.out_row_base + row0[tc.g] + local;
       long long dest = out_row;
       float sc = 1.0f;
       if (EPI == EPI_SCATTER && valid) {
         dest = p.perm ? p.perm[out_row] : out_row;
-        if (p.scale) sc = p.scale[dest];
+        if (dest < 0 || dest >= p.row_limit) {
+          atomicOr(&g_tc_error, 2u);
+          valid = false;
+          dest = 0;
+        } else if (p.scale) {
+          sc = p.scale[dest];
+        }
       }
       // EPI_REPLICATE: this row's destinations, read once per tile.
       int rdst[8];
@@ -807,6 +823,7 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   }
   p.partial = a.partial;
   p.part_rows = a.part_rows;
+  p.row_limit = a.max_rows > 0 ? a.max_rows : (1LL << 62);
   const long long m_tiles_max = a.max_rows / C::TILE_M + a.G;
   long long tiles = m_tiles_max * p.n_tiles_n * p.split_k;
   if (PAIR) {

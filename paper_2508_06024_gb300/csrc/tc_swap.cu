@@ -30,7 +30,9 @@
 
 namespace ec2moe {
 
-__device__ unsigned int g_swap_error;  // bit 0: a bounded wait timed out
+// bit 0: a bounded wait timed out; bit 1: a group range (offsets) or a
+// scatter destination (perm) outside the rows of the call was skipped
+__device__ unsigned int g_swap_error;
 
 namespace {
 
@@ -76,6 +78,7 @@ struct SwParams {
   int split_k, kb_per_split;
   int n_blk;  // weight tiles per group along N
   long long timeout;
+  long long row_limit;  // rows of the call: group ranges and scatter destinations lie in [0, row_limit)
 };
 
 struct SwUnit {
@@ -143,6 +146,12 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
         if (p.offsets) {
           r0v[c] = p.offsets[g];
           mgv[c] = p.offsets[g + 1] - r0v[c];
+          if (r0v[c] < 0 || mgv[c] < 0 || static_cast<long long>(r0v[c]) + mgv[c] > p.row_limit) {
+            // not a range of this call's rows: the group is skipped
+            atomicOr(&g_swap_error, 2u);
+            r0v[c] = 0;
+            mgv[c] = 0;
+          }
         } else {
           r0v[c] = g * p.M;
           mgv[c] = p.M;
@@ -347,6 +356,10 @@ __global__ void __launch_bounds__(SW_THREADS, 1)
             if (EPI == EPI_GELU) y = gelu_bf16out(y);
             if (EPI == EPI_SCATTER) {
               dest = p.perm ? p.perm[out_row] : out_row;
+              if (dest < 0 || dest >= p.row_limit) {
+                atomicOr(&g_swap_error, 2u);
+                continue;
+              }
               if (p.scale) y *= p.scale[dest];
             }
             o[dest * p.ldo + col] = __float2bfloat16_rn(y);
@@ -450,6 +463,7 @@ cudaError_t launch_gemm_swap(const GemmArgs& a, int epi, cudaStream_t s) {
   p.partial = a.partial;
   p.part_rows = a.part_rows;
   p.timeout = a.timeout_cycles;
+  p.row_limit = a.max_rows > 0 ? a.max_rows : (1LL << 62);
   p.n_blk = static_cast<int>((a.N + tn - 1) / tn);
   p.split_k = epi == EPI_PARTIAL ? a.split_k : 1;
   const int num_kb = (a.K + SW_BK - 1) / SW_BK;

@@ -102,3 +102,64 @@ def test_route_out_of_range_ids_are_skipped_and_reported(T, k, E, noalloc):
         C.ec2moe_route(desc, idx, counts, offsets, perm, inv, X, d, dst, ws, wsb)
     assert C.ec2moe_last_device_error() == C.OK
     assert int(counts.sum().item()) == n
+
+
+# Expert-order tables handed to ec2moe_experts that do not describe the call's
+# rows: every grouped GEMM (swapped-operand kernel for <= 16 rows, tensor-core
+# kernel, SIMT kernel for fp32) checks each group range against the rows and
+# each scatter destination, skips what lies outside, and reports
+# EC2MOE_ERR_INVALID_ARG; nothing past the output buffer is written.
+EXPERT_SHAPES = [(8, 2, 4, 256, 256, C.BF16), (200, 2, 4, 256, 512, C.BF16), (96, 2, 4, 128, 256, C.F32)]
+CORRUPTIONS = ["offset-past-rows", "negative-offset", "decreasing-offsets", "perm-out-of-range"]
+
+
+@pytest.mark.parametrize("shape", EXPERT_SHAPES, ids=["swapped", "tensor-core", "simt-fp32"])
+@pytest.mark.parametrize("bad", CORRUPTIONS)
+def test_experts_skip_tables_outside_the_rows(shape, bad):
+    T, k, E, d, d_ff, dtype = shape
+    n = T * k
+    dt = torch.bfloat16 if dtype == C.BF16 else torch.float32
+    g = torch.Generator(device="cuda")
+    g.manual_seed(77 + T)
+    Xp = torch.randn(n, d, generator=g, device="cuda").to(dt)
+    W1 = (torch.randn(E, d_ff, d, generator=g, device="cuda") * d ** -0.5).to(dt)
+    W3 = (torch.randn(E, d_ff, d, generator=g, device="cuda") * d ** -0.5).to(dt)
+    W2 = (torch.randn(E, d, d_ff, generator=g, device="cuda") * d_ff ** -0.5).to(dt)
+    rs = np.random.default_rng(T)
+    counts = np.bincount(rs.integers(0, E, size=n), minlength=E)
+    counts[1] = max(counts[1], 2)
+    counts[E - 1] = max(counts[E - 1], 1)
+    counts[0] = n - counts[1:].sum()
+    assert counts[0] >= 1
+    offsets_h = np.concatenate([[0], np.cumsum(counts)]).astype(np.int32)
+    perm_h = rs.permutation(n).astype(np.int32)
+    w = torch.from_numpy(rs.uniform(0.1, 1.0, size=(T, k)).astype(np.float32)).cuda()
+    desc = C.make_desc(T=T, d=d, E=E, d_ff=d_ff, k=k, act=C.SWIGLU, dtype=dtype)
+    ews = C.ec2moe_experts_workspace_size(desc)
+    ew = torch.empty(max(ews, 16), dtype=torch.uint8, device="cuda")
+    guard = 8
+
+    def call(offs, perm):
+        slot = torch.full((n + guard, d), 7.0, dtype=dt, device="cuda")
+        C.ec2moe_experts(desc, Xp, torch.from_numpy(offs).cuda(), W1, W3, W2, w, torch.from_numpy(perm).cuda(),
+                         slot, ew, ews)
+        return slot, C.ec2moe_last_device_error()
+
+    ref, status = call(offsets_h, perm_h)
+    assert status == C.OK
+    assert torch.all(ref[n:] == 7.0)
+    offs, perm = offsets_h.copy(), perm_h.copy()
+    if bad == "offset-past-rows":
+        offs[E] = n + 100
+    elif bad == "negative-offset":
+        offs[1] = -5
+    elif bad == "decreasing-offsets":
+        offs[2] = offs[1] - 1
+    else:
+        perm[3] = n + 1000
+    out, status = call(offs, perm)
+    assert status == C.ERR_INVALID_ARG
+    assert torch.all(out[n:] == 7.0)  # nothing written past the rows
+    again, status = call(offsets_h, perm_h)
+    assert status == C.OK
+    assert torch.equal(again, ref)
