@@ -49,6 +49,17 @@ namespace {
 //                tile add the bias and take the token's softmax / Top-k
 //                decision (decide_token_thread);
 //   warps 2..13  on the layer path, reserve the tile's rows per expert.
+// With d_model of 2048 or more (32 or more stages per tile) a tile belongs to
+// a cluster of GC_CS CTAs on as many SMs instead: CTA c of the cluster runs
+// the stages [c nk / GC_CS, (c + 1) nk / GC_CS) and owns the decisions of
+// rows [c 128 / GC_CS, (c + 1) 128 / GC_CS).  Each drain thread sends its
+// row's partial logits to the row's owner (st.async into the owner's shared
+// memory, counted on the owner's receive barrier), and the owner adds the
+// cluster's partials in CTA order before the bias and the decision; every CTA
+// reserves the rows it decided.  One tile per cluster: such grids are one
+// cluster per tile, run in waves when they exceed the SMs.  A tile's reading
+// of X is then spread over twice the SMs (the per-SM copy rate, not HBM,
+// bounds a 128-token tile's stream).
 // Every mbarrier wait is bounded; on a timeout the error word is set, copies
 // and MMAs in flight are drained and the CTA finishes its tiles without
 // waiting (the decisions then see garbage logits but still name valid experts).
@@ -60,26 +71,32 @@ constexpr int GC_MAX_STAGES = 10;
 constexpr int GC_THREADS = 448;
 constexpr int GC_WORKERS = 384;     // warps 2..13
 constexpr int GC_ACC_STRIDE = 256;  // TMEM columns between the two accumulators (3 * O_pad <= 240 each)
+constexpr int GC_CS = 2;            // CTAs per tile (cluster) when d_model is split
+constexpr int GC_SPLIT_MIN_NK = 32; // stages per tile from which d_model is split
 
 struct GcLayout {
-  int n_pad, O, k, E, stages;
+  int n_pad, O, k, E, stages, cs;
   int stage_bytes, w3_off, raw_off;
   int log_stride;  // logits row of a token: O logits + 16 group scratch words, odd (conflict-free rows)
-  int log_off, idx_off, tab_off, base_off, bias_off, bar_off, total;
-  __host__ __device__ GcLayout(int O_, int k_, int E_, int stages_, bool prep)
-      : O(O_), k(k_), E(E_), stages(stages_) {
+  int rstride;     // floats per received partial-logit row: n_pad + 4 (16-byte rows, shifted banks)
+  int log_off, idx_off, tab_off, base_off, bias_off, recv_off, bar_off, total;
+  __host__ __device__ GcLayout(int O_, int k_, int E_, int stages_, bool prep, int cs_)
+      : O(O_), k(k_), E(E_), stages(stages_), cs(cs_) {
     n_pad = (O + 15) / 16 * 16;
     w3_off = GC_BM * GC_BK * 2;
     raw_off = w3_off + 3 * n_pad * 128;
     stage_bytes = raw_off + (prep ? 0 : n_pad * 256);  // a multiple of 1024
     log_stride = (O + 16) | 1;
+    rstride = n_pad + 4;
     log_off = stages * stage_bytes;
     idx_off = log_off + GC_BM * log_stride * 4;
     tab_off = idx_off + GC_BM * k * 4;
     base_off = tab_off + (GC_BM * k / 32) * E * 4;
     bias_off = base_off + 4 * E;
-    bar_off = (bias_off + 4 * O + 7) / 8 * 8;
-    total = bar_off + (3 * stages + 5) * 8 + 16;
+    // received partials: [source CTA][owned row][rstride] (cs > 1)
+    recv_off = (bias_off + 4 * O + 15) / 16 * 16;
+    bar_off = (recv_off + (cs > 1 ? GC_BM * rstride * 4 : 0) + 7) / 8 * 8;
+    total = bar_off + (3 * stages + 6) * 8 + 16;
   }
 };
 
@@ -87,6 +104,7 @@ struct GcParams {
   KParams kp;
   int n_pad;
   int stages;
+  int cs;  // CTAs per tile (cluster size); 1 = one CTA per tile, persistent over tiles
   long long timeout;
 };
 
@@ -328,18 +346,21 @@ __device__ __forceinline__ void decide_k1_regs(const float (&x)[NB][16], int E, 
     }
 }
 
-// Rows of the tile reserved per expert (the layer path), with the worker warps
-// only: entry i of the tile (token i / k, slot i % k) gets route_rel = the
-// expert's reserved base + the number of earlier entries of the tile with the
-// same expert.  32-entry chunks are ranked with a warp match, chunk counts are
-// turned into per-expert prefixes, and one atomicAdd per expert reserves the
-// tile's rows.
-__device__ void route_tile_workers(const KParams& p, int tile, const int* sIdx, int* sTab, int* s_base, int wt) {
+// Rows [row_lo, row_lo + n_rows) of the tile reserved per expert (the layer
+// path), with the worker warps only: entry i of the range (token row_lo + i /
+// k of the tile, slot i % k) gets route_rel = the expert's reserved base + the
+// number of earlier entries of the range with the same expert.  sIdx holds the
+// range's decisions.  32-entry chunks are ranked with a warp match, chunk
+// counts are turned into per-expert prefixes, and one atomicAdd per expert
+// reserves the range's rows.
+__device__ void route_tile_workers(const KParams& p, int tile, int row_lo, int n_rows, const int* sIdx, int* sTab,
+                                   int* s_base, int wt) {
   const int wi = wt >> 5, lane = wt & 31;
-  const int nt = GC_BM * p.k;
-  const long long e0 = (long long)tile * nt;
+  const int nt = n_rows * p.k;
+  const long long e0 = ((long long)tile * GC_BM + row_lo) * p.k;
   const long long n = (long long)p.T * p.k;
-  const int live = (int)((n - e0) < nt ? (n - e0) : nt);
+  const long long rem = n - e0;
+  const int live = rem <= 0 ? 0 : (int)(rem < nt ? rem : nt);
   const int nch = (live + 31) / 32;
   constexpr int NW = GC_WORKERS / 32;
   constexpr int MAXC = (GC_BM * MAX_TOPK / 32 + NW - 1) / NW;
@@ -433,20 +454,23 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int nglob = (p.K == 1) ? 0 : p.K;
   const int O = p.E + nglob;
-  const GcLayout L(O, p.k, p.E, gp.stages, PREP);
+  const int cs = gp.cs;
+  const GcLayout L(O, p.k, p.E, gp.stages, PREP, cs);
   const int S = gp.stages;
   float* sLog = reinterpret_cast<float*>(smem + L.log_off);
   int* sIdx = reinterpret_cast<int*>(smem + L.idx_off);
   int* sTab = reinterpret_cast<int*>(smem + L.tab_off);
   int* s_base = reinterpret_cast<int*>(smem + L.base_off);
   float* s_bias = reinterpret_cast<float*>(smem + L.bias_off);
+  float* s_recv = reinterpret_cast<float*>(smem + L.recv_off);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L.bar_off);
   uint64_t* conv = full + S;
   uint64_t* empty = conv + S;
   uint64_t* tfull = empty + S;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* recvb = drain + 1;  // partial logits from the other CTAs of the cluster (cs > 1)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(recvb + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -455,6 +479,14 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
   const int nk = (p.d + GC_BK - 1) / GC_BK;
   const long long budget = gp.timeout;
   const int n_pad = gp.n_pad;
+  // cs > 1: cluster `tile` of cs CTAs (one tile per cluster); this CTA runs
+  // stages [kb_lo, kb_lo + cnt) and decides rows [rank * rows_own, ...)
+  const int rank = cs > 1 ? static_cast<int>(cluster_ctarank()) : 0;
+  const int tile_first = cs > 1 ? static_cast<int>(cluster_id_x()) : static_cast<int>(blockIdx.x);
+  const int tile_step = cs > 1 ? static_cast<int>(cluster_count_x()) : static_cast<int>(gridDim.x);
+  const int kb_lo = rank * nk / cs;
+  const int cnt = (rank + 1) * nk / cs - kb_lo;
+  const int rows_own = GC_BM / cs;
   pdl_trigger();
 
   if (threadIdx.x == 0) {
@@ -468,9 +500,12 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
       mbar_init(smem_u32(&tempty[a]), 4);
     }
     mbar_init(smem_u32(drain), 1);
+    mbar_init(smem_u32(recvb), 1);
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    // the owned rows' partials of the other cs - 1 CTAs (one tile per cluster)
+    if (cs > 1) mbar_expect_tx(smem_u32(recvb), static_cast<uint32_t>((cs - 1) * rows_own * n_pad * 4));
   }
   for (int o = threadIdx.x - 64; o >= 0 && o < O; o += GC_THREADS - 64)
     s_bias[o] = o < p.E ? p.b_local[o] : p.b_global[o - p.E];
@@ -487,6 +522,8 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
   }
   tc_fence_before();
   __syncthreads();
+  // every receive barrier of the cluster is initialised before any partial is sent
+  if (cs > 1) cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -498,11 +535,11 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
     if (lane == 0) {
       const uint32_t xbytes = GC_BM * GC_BK * 2;
       const uint32_t wbytes = PREP ? 3 * n_pad * GC_BK * 2 : O * GC_BK * 4;
-      const int my_tiles = blockIdx.x < n_tiles ? (n_tiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
-      const int total = my_tiles * nk;
+      const int my_tiles = tile_first < n_tiles ? (n_tiles - 1 - tile_first) / tile_step + 1 : 0;
+      const int total = my_tiles * cnt;
       const int pre = PREP ? (total < S ? total : S) : 0;
       auto load_w = [&](int c, uint8_t* st, uint32_t fb) {
-        const int kc = c % nk;
+        const int kc = kb_lo + c % cnt;
         if (PREP) {
           tma_load_2d(smem_u32(st + L.w3_off), &tmW, kc * GC_BK, 0, fb);
         } else {
@@ -513,8 +550,8 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
       for (int c = 0; c < pre; ++c) {
         const uint32_t fb = smem_u32(&full[c]);
         mbar_expect_tx(fb, xbytes + wbytes);
-        tma_load_2d(smem_u32(smem + c * L.stage_bytes), &tmX, (c % nk) * GC_BK,
-                    (blockIdx.x + (c / nk) * gridDim.x) * GC_BM, fb);
+        tma_load_2d(smem_u32(smem + c * L.stage_bytes), &tmX, (kb_lo + c % cnt) * GC_BK,
+                    (tile_first + (c / cnt) * tile_step) * GC_BM, fb);
       }
       pdl_wait();
       for (int c = 0; c < pre; ++c) load_w(c, smem + c * L.stage_bytes, smem_u32(&full[c]));
@@ -530,7 +567,8 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
         uint8_t* st = smem + stage * L.stage_bytes;
         const uint32_t fb = smem_u32(&full[stage]);
         mbar_expect_tx(fb, xbytes + wbytes);
-        tma_load_2d(smem_u32(st), &tmX, (c % nk) * GC_BK, (blockIdx.x + (c / nk) * gridDim.x) * GC_BM, fb);
+        tma_load_2d(smem_u32(st), &tmX, (kb_lo + c % cnt) * GC_BK, (tile_first + (c / cnt) * tile_step) * GC_BM,
+                    fb);
         load_w(c, st, fb);
         issued |= 1u << stage;
         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
@@ -553,8 +591,8 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
       int acc = 0;
       uint32_t uses0 = 0, uses1 = 0;
       bool ok = true, any = false;
-      for (int tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-        for (int seg = 0; seg < nk && ok; seg += GC_SEG) {
+      for (int tile = tile_first; tile < n_tiles && ok; tile += tile_step) {
+        for (int seg = 0; seg < cnt && ok; seg += GC_SEG) {
           const uint32_t uses = acc ? uses1 : uses0;
           if (!mbar_wait(smem_u32(&tempty[acc]), (uses & 1u) ^ 1u, budget, abort_flag, &g_gate_error)) {
             ok = false;
@@ -562,7 +600,7 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
           }
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + acc * GC_ACC_STRIDE;
-          const int seg_end = seg + GC_SEG < nk ? seg + GC_SEG : nk;
+          const int seg_end = seg + GC_SEG < cnt ? seg + GC_SEG : cnt;
           for (int kc = seg; kc < seg_end; ++kc) {
             if ((!PREP && !mbar_wait(smem_u32(&conv[stage]), phase, budget, abort_flag, &g_gate_error)) ||
                 !mbar_wait(smem_u32(&full[stage]), phase, budget, abort_flag, &g_gate_error)) {
@@ -609,14 +647,14 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
     int acc_sel = 0;
     uint32_t uses0 = 0, uses1 = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
+    for (int tile = tile_first; tile < n_tiles; tile += tile_step) {
       if (is_drain) {
         float acc[NB][16];
 #pragma unroll
         for (int b = 0; b < NB; ++b)
 #pragma unroll
           for (int j = 0; j < 16; ++j) acc[b][j] = 0.0f;
-        for (int seg = 0; seg < nk; seg += GC_SEG) {
+        for (int seg = 0; seg < cnt; seg += GC_SEG) {
           const uint32_t uses = acc_sel ? uses1 : uses0;
           if (ok) ok = mbar_wait(smem_u32(&tfull[acc_sel]), uses & 1u, budget, abort_flag, &g_gate_error);
           if (ok) {
@@ -641,43 +679,79 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
           else ++uses0;
           acc_sel ^= 1;
         }
+        bool decide_here = true;
+        if (cs > 1) {
+          // this row's partial logits go to the CTA that owns its decision;
+          // the owner adds the cluster's partials in CTA order
+          const int owner = row / rows_own;
+          const int lrow = row - owner * rows_own;
+          if (owner != rank) {
+            decide_here = false;
+            if (ok) {
+              const uint32_t dst = map_to_rank(smem_u32(s_recv + (rank * rows_own + lrow) * L.rstride), owner);
+              const uint32_t rb = map_to_rank(smem_u32(recvb), owner);
 #pragma unroll
-        for (int b = 0; b < NB; ++b)
+              for (int b = 0; b < NB; ++b)
+                if (b * 16 < n_pad)
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const int o = b * 16 + j;
-            if (o < O) acc[b][j] += s_bias[o];
+                  for (int j = 0; j < 16; j += 4)
+                    st_async_v4(dst + (b * 16 + j) * 4, acc[b][j], acc[b][j + 1], acc[b][j + 2], acc[b][j + 3], rb);
+            }
+          } else {
+            if (ok) ok = mbar_wait_cluster(smem_u32(recvb), 0, budget, abort_flag, &g_gate_error);
+            if (ok) {
+#pragma unroll
+              for (int b = 0; b < NB; ++b)
+                if (b * 16 < n_pad)
+#pragma unroll
+                  for (int j = 0; j < 16; ++j) {
+                    float t = rank == 0 ? acc[b][j] : s_recv[lrow * L.rstride + b * 16 + j];
+                    for (int c = 1; c < cs; ++c)
+                      t += c == rank ? acc[b][j] : s_recv[(c * rows_own + lrow) * L.rstride + b * 16 + j];
+                    acc[b][j] = t;
+                  }
+            }
           }
-        const int tok = tile * GC_BM + row;
-        int* sx = p.route_counts ? sIdx + row * p.k : nullptr;
-        if (!nglob) {
-          if (tok < p.T) {
-            if (p.k == 1) decide_k1_regs<NB, 1>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
-            else if (p.k == 2) decide_k1_regs<NB, 2>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
-            else if (p.k <= 4) decide_k1_regs<NB, 4>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
-            else decide_k1_regs<NB, 8>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
-          }
-        } else {
-          float* Lrow = sLog + row * L.log_stride;
+        }
+        if (decide_here) {
 #pragma unroll
           for (int b = 0; b < NB; ++b)
 #pragma unroll
             for (int j = 0; j < 16; ++j) {
               const int o = b * 16 + j;
-              if (o < O) Lrow[o] = acc[b][j];
+              if (o < O) acc[b][j] += s_bias[o];
             }
-          if (tok < p.T) {
-            if (p.k == 1) decide_token_thread<1>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
-            else if (p.k == 2) decide_token_thread<2>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
-            else if (p.k <= 4) decide_token_thread<4>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
-            else decide_token_thread<8>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+          const int tok = tile * GC_BM + row;
+          int* sx = p.route_counts ? sIdx + row * p.k : nullptr;
+          if (!nglob) {
+            if (tok < p.T) {
+              if (p.k == 1) decide_k1_regs<NB, 1>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
+              else if (p.k == 2) decide_k1_regs<NB, 2>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
+              else if (p.k <= 4) decide_k1_regs<NB, 4>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
+              else decide_k1_regs<NB, 8>(acc, p.E, p.k, p.renorm, mregs, p.topk_idx, p.topk_w, tok, sx);
+            }
+          } else {
+            float* Lrow = sLog + row * L.log_stride;
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const int o = b * 16 + j;
+                if (o < O) Lrow[o] = acc[b][j];
+              }
+            if (tok < p.T) {
+              if (p.k == 1) decide_token_thread<1>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+              else if (p.k == 2) decide_token_thread<2>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+              else if (p.k <= 4) decide_token_thread<4>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+              else decide_token_thread<8>(p.E, p.K, p.k, p.renorm, p.top_groups, mregs, Lrow, Lrow + O, p.topk_idx, p.topk_w, tok, sx);
+            }
           }
-        }
+        }  // decide_here
       } else if (!PREP) {
         // split the raw fp32 gate rows of each stage into three bf16 terms,
         // written in the swizzled K-major layout of the B operand
         const int ct = threadIdx.x - 192;
-        for (int kc = 0; kc < nk; ++kc) {
+        for (int kc = 0; kc < cnt; ++kc) {
           if (ok) ok = mbar_wait(smem_u32(&full[stage]), phase, budget, abort_flag, &g_gate_error);
           if (ok) {
             uint8_t* st = smem + stage * L.stage_bytes;
@@ -714,7 +788,7 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
       }
       if (p.route_counts) {
         asm volatile("bar.sync 1, %0;" ::"r"(GC_WORKERS) : "memory");
-        route_tile_workers(p, tile, sIdx, sTab, s_base, wt);
+        route_tile_workers(p, tile, rank * rows_own, rows_own, sIdx + rank * rows_own * p.k, sTab, s_base, wt);
       }
     }
     tc_fence_before();
@@ -722,47 +796,83 @@ __global__ void __launch_bounds__(GC_THREADS, 1)
 
   tc_fence_before();
   __syncthreads();
+  // no CTA of the cluster leaves while partials to or from it are in flight
+  if (cs > 1) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(512) : "memory");
   }
 }
 
-// Stages that fit next to the logits and routing tables.
-int gc_stages(int O, int k, int E, bool prep) {
+// Stages that fit next to the logits, routing tables and received partials.
+int gc_stages(int O, int k, int E, bool prep, int cs) {
   for (int s = GC_MAX_STAGES; s >= 2; --s)
-    if (GcLayout(O, k, E, s, prep).total + 1024 <= 232448) return s;
+    if (GcLayout(O, k, E, s, prep, cs).total + 1024 <= 232448) return s;
   return 0;
 }
 
+// CTAs per tile: d_model is split over a cluster of GC_CS when a tile has at
+// least GC_SPLIT_MIN_NK stages and the received partials still leave four
+// pipeline stages (counted for the larger, self-splitting layout), whatever
+// the token count and whether the rows come prepared, so every call of one
+// layer shape sums its logits in the same order.
+int gc_cluster_size(int O, int k, int E, int d) {
+  if ((d + GC_BK - 1) / GC_BK < GC_SPLIT_MIN_NK) return 1;
+  return gc_stages(O, k, E, false, GC_CS) >= 4 ? GC_CS : 1;
+}
+
+// CTAs the gate kernel launches (cs > 1: a cluster per tile, run in waves
+// when they exceed the SMs; cs = 1: persistent, at most one per SM).
+int gc_blocks(int T, int cs) {
+  const int n_tiles = (T + GC_BM - 1) / GC_BM;
+  if (cs > 1) return n_tiles * cs;
+  return n_tiles < sm_count() ? n_tiles : sm_count();
+}
+
 template <int NB, bool PREP>
-cudaError_t launch_gate_tc_nb(const KParams& p, int stages, cudaStream_t s, const CUtensorMap& mX,
+cudaError_t launch_gate_tc_nb(const KParams& p, int stages, int cs, cudaStream_t s, const CUtensorMap& mX,
                               const CUtensorMap& mW, const CUtensorMap& mWg) {
   const int O = p.E + (p.K == 1 ? 0 : p.K);
   GcParams gp;
   gp.kp = p;
   gp.n_pad = (O + 15) / 16 * 16;
   gp.stages = stages;
+  gp.cs = cs;
   gp.timeout = default_timeout_cycles();
-  const int smem = GcLayout(O, p.k, p.E, stages, PREP).total + 1024;
+  const int smem = GcLayout(O, p.k, p.E, stages, PREP, cs).total + 1024;
   cudaError_t e = ensure_smem_attr(reinterpret_cast<const void*>(gate_tc_kernel<NB, PREP>), smem);
   if (e != cudaSuccess) return e;
-  const int n_tiles = (p.T + GC_BM - 1) / GC_BM;
-  const int blocks = n_tiles < sm_count() ? n_tiles : sm_count();
-  return launch_kernel(gate_tc_kernel<NB, PREP>, dim3(blocks), dim3(GC_THREADS), (size_t)smem, s, mX, mW, mWg, gp);
+  const int blocks = gc_blocks(p.T, cs);
+  if (cs == 1)
+    return launch_kernel(gate_tc_kernel<NB, PREP>, dim3(blocks), dim3(GC_THREADS), (size_t)smem, s, mX, mW, mWg, gp);
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(blocks);
+  cfg.blockDim = dim3(GC_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cs;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = next_launch_pdl() ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, gate_tc_kernel<NB, PREP>, mX, mW, mWg, gp);
 }
 
 template <bool PREP>
-cudaError_t launch_gate_tc(const KParams& p, int stages, cudaStream_t s, const CUtensorMap& mX,
+cudaError_t launch_gate_tc(const KParams& p, int stages, int cs, cudaStream_t s, const CUtensorMap& mX,
                            const CUtensorMap& mW, const CUtensorMap& mWg) {
   const int O = p.E + (p.K == 1 ? 0 : p.K);
   // NB = accumulator blocks of 16 gate rows a drain thread keeps; 3 and 4
   // run as 5 (the extra blocks read allocated TMEM columns past the gate rows
   // and are never used), which keeps the number of kernel variants small.
   switch ((O + 15) / 16) {
-    case 1: return launch_gate_tc_nb<1, PREP>(p, stages, s, mX, mW, mWg);
-    case 2: return launch_gate_tc_nb<2, PREP>(p, stages, s, mX, mW, mWg);
-    default: return launch_gate_tc_nb<5, PREP>(p, stages, s, mX, mW, mWg);
+    case 1: return launch_gate_tc_nb<1, PREP>(p, stages, cs, s, mX, mW, mWg);
+    case 2: return launch_gate_tc_nb<2, PREP>(p, stages, cs, s, mX, mW, mWg);
+    default: return launch_gate_tc_nb<5, PREP>(p, stages, cs, s, mX, mW, mWg);
   }
 }
 
@@ -785,7 +895,8 @@ cudaError_t launch_gate_tensor(const GateArgs& a, KParams p, int O, bool bf16, c
   if (bf16 && !simt_only && O <= GC_MAX_O && a.d % 8 == 0 && a.T > 0 && w_aligned) {
     const bool prep = a.w_split != nullptr;
     const int n_pad = (O + 15) / 16 * 16;
-    const int stages = gc_stages(O, a.k, a.E, prep);
+    const int cs = gc_cluster_size(O, a.k, a.E, a.d);
+    const int stages = gc_stages(O, a.k, a.E, prep, cs);
     CUtensorMap mX, mW, mWg;
     bool maps = stages >= 2 && make_tensor_map_bf16(&mX, a.X, a.T, a.d, GC_BM);
     if (prep) {
@@ -818,10 +929,11 @@ cudaError_t launch_gate_tensor(const GateArgs& a, KParams p, int O, bool bf16, c
       }
       KernelScope ks("gate_topk", s);
       if (held_sms) {  // one CTA per SM (the kernel's shared memory allows no second)
-        const int n_tiles = (a.T + GC_BM - 1) / GC_BM;
-        *held_sms = n_tiles < sm_count() ? n_tiles : sm_count();
+        const int b = gc_blocks(a.T, cs);
+        *held_sms = b < sm_count() ? b : sm_count();
       }
-      e = prep ? launch_gate_tc<true>(p, stages, s, mX, mW, mWg) : launch_gate_tc<false>(p, stages, s, mX, mW, mWg);
+      e = prep ? launch_gate_tc<true>(p, stages, cs, s, mX, mW, mWg)
+               : launch_gate_tc<false>(p, stages, cs, s, mX, mW, mWg);
       if (e != cudaSuccess) return e;
       return cudaGetLastError();
     }

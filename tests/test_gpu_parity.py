@@ -60,6 +60,13 @@ GATE_CASES = [
     S.preset("switch_bf16", T=300, d=200, seed=16),
     S.preset("finegrained_bf16", T=900, n_groups=16, k=4, seed=19),
     S.preset("finegrained_bf16", T=700, E=128, n_groups=8, n_allowed=64, k=4, seed=15),
+    # d_model split over a two-CTA cluster per tile (d_model >= 2048): a
+    # ragged last tile (104 rows, the second CTA owning rows 64..103), a
+    # single tile with 6 rows in the second CTA's half, and the one-group
+    # decision (K = 1, Top-2) over five tiles
+    S.preset("mixtral_bf16", T=1000, seed=71),
+    S.preset("mixtral_bf16", T=70, seed=72),
+    S.preset("decode_bf16", T=600, n_allowed=6, seed=73),
 ]
 
 
@@ -232,6 +239,11 @@ LAYER_CASES = [
     (S.preset("finegrained_bf16", T=150, seed=63), None),
     (S.preset("tiny_fp32", T=100, d=1024, seed=52), None),
     (S.preset("tiny_fp32", T=7, seed=45), None),
+    # the gate's two-CTA clusters with the fused row reservations: a last tile
+    # of 44 tokens (the second CTA owns no token of it), and K = 1 over five
+    # tiles
+    (S.preset("mixtral_bf16", T=300, d_ff=1024, seed=74), None),
+    (S.preset("decode_bf16", T=520, n_allowed=8, d_ff=1024, r=128, seed=75), None),
     # the limits: 128 experts in 16 groups, Top-8, 144 gate rows; and many
     # tiles per CTA in every kernel
     (S.preset("switch_bf16", T=1024, d=512, E=128, d_ff=512, n_groups=16, k=8, n_allowed=96, r=128, seed=47), 256),

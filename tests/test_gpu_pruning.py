@@ -42,6 +42,7 @@ PRUNE_CASES = [
     S.preset("finegrained_bf16", T=777, top_groups=3, seed=73),
     S.preset("finegrained_bf16", T=600, top_groups=3, k=4, renorm_topk=1, seed=74),
     S.preset("mixtral_bf16", T=129, d_ff=1024, top_groups=1, n_allowed=8, seed=75),
+    S.preset("mixtral_bf16", T=300, d_ff=1024, top_groups=1, n_allowed=8, seed=79),
     S.preset("tiny_fp32", T=256, n_allowed=8, top_groups=1, seed=76),
     S.preset("switch_bf16", T=300, E=16, n_groups=4, k=2, n_allowed=16, top_groups=4, seed=77),
 ]

@@ -11,8 +11,9 @@ compared bit for bit with no near-tie exclusion for the designed ties.  Tokens
 excluded are only those with an accidental near-tie (< 1e-6 in log g) between
 two experts that are not twins; the test also checks that the designed ties
 decide many tokens.  Both ec2moe_gate and the layer call are checked, on the
-tensor-core gate (bf16), the small-batch split-d gate (<= 256 tokens,
-d_model >= 1024) and the SIMT gate (fp32).  Twin experts also get identical
+tensor-core gate (bf16; two CTAs per tile at d_model >= 2048), the
+small-batch split-d gate (<= 256 tokens, d_model >= 1024) and the SIMT gate
+(fp32).  Twin experts also get identical
 expert weights, so the layer's output is checked against the oracle whichever
 twin each side picks.
 """
@@ -111,6 +112,7 @@ TIE_CASES = [
     (S.preset("switch_bf16", T=777, E=16, k=3, n_groups=4, seed=63), "groups"),
     (S.preset("finegrained_bf16", T=600, seed=64), "groups"),
     (S.preset("mixtral_bf16", T=129, d_ff=1024, seed=65), "groups"),
+    (S.preset("mixtral_bf16", T=400, d_ff=1024, seed=67), "groups"),
     (S.preset("tiny_fp32", T=200, seed=66), "groups"),
 ]
 
