@@ -181,6 +181,29 @@ def roofline_for(cfg, name, avg_ms, peaks, peaks_src, traffic, touched: int = 0)
             "algorithmic_bytes": byts, "avg_ms": round(avg_ms, 5)}
 
 
+def stream_reference_ms(torch, dev, stream, flush, nbytes: float, reps: int) -> float:
+    """Mean device time of one torch launch that reads `nbytes` (an int64 max
+    over a buffer of that size), bracketed by an event pair on the stream with
+    L2 flushed first, as each library kernel is.  A sleep kernel ahead of the
+    first event keeps the host's enqueue time out of the bracket.  This is what
+    a plain stream of the same bytes costs in one launch, ramp and tail
+    included: the reference point for kernels whose roofline is HBM."""
+    buf = torch.ones(max(1, int(nbytes) // 8), dtype=torch.int64, device=dev)
+    times = []
+    for i in range(reps + 1):
+        flush()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(100000)
+        a.record(stream)
+        buf.max()
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        if i:
+            times.append(a.elapsed_time(b))
+    del buf
+    return statistics.mean(times)
+
+
 def committed_traffic(cfg, kernel):
     """dram read+write bytes per launch for (workload, kernel) from profiles/traffic.txt, or None.
 
@@ -616,6 +639,14 @@ def run_ours(args):
     others = {n: roofline_for(cfg, n, kern[n]["avg_ms"], peaks, peaks_src, committed_traffic(cfg, n), touched)
               for n in kern}
     layer_flops = sum(kernel_work(cfg, n)[0] * kern[n]["launches_per_step"] for n in kern)
+    # HBM-bound kernels beside a plain one-launch read of their algorithmic bytes
+    for n in kern:
+        if others[n]["bound"] == "hbm" and others[n]["algorithmic_bytes"] >= (1 << 20):
+            sm = stream_reference_ms(torch, dev, stream, flush, others[n]["algorithmic_bytes"], prof_steps)
+            kern[n]["stream_ms"] = round(sm, 5)
+            kern[n]["vs_stream"] = round(sm / kern[n]["avg_ms"], 3)
+    if "stream_ms" in kern[dominant]:
+        roof["stream_ms"] = kern[dominant]["stream_ms"]
 
     cpu = None
     if not args.no_cpu_baseline and world == 1:
@@ -636,7 +667,9 @@ def run_ours(args):
                              "together larger than L2)",
                    "parallelism": f"token-parallel replicas x{world}",
                    "kernel_timing": "per launch index, a graph of the whole call with only that launch bracketed "
-                                    "by CUDA events, L2 flushed; share = kernel time / step time"},
+                                    "by CUDA events, L2 flushed; share = kernel time / step time; stream_ms = one "
+                                    "torch launch reading the kernel's algorithmic bytes, bracketed the same way "
+                                    "(HBM-bound kernels); vs_stream = stream_ms / avg_ms"},
         "layer_tflops": round(layer_flops / (t_step * 1e-3) / 1e12, 2),
         "layer_frac_bf16_peak": round(layer_flops / (t_step * 1e-3) / 1e12 / peaks["bf16_tflops"], 4),
         "roofline": roof,

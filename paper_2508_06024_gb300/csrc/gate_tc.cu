@@ -816,8 +816,14 @@ int gc_stages(int O, int k, int E, bool prep, int cs) {
 // pipeline stages (counted for the larger, self-splitting layout), whatever
 // the token count and whether the rows come prepared, so every call of one
 // layer shape sums its logits in the same order.
+// EC2MOE_GATE_SPLIT_MIN_STAGES=n in the environment moves the threshold
+// (A/B comparisons; the split computes the same logits up to summation order).
 int gc_cluster_size(int O, int k, int E, int d) {
-  if ((d + GC_BK - 1) / GC_BK < GC_SPLIT_MIN_NK) return 1;
+  static const int min_nk = [] {
+    const char* v = getenv("EC2MOE_GATE_SPLIT_MIN_STAGES");
+    return v && atoi(v) > 0 ? atoi(v) : GC_SPLIT_MIN_NK;
+  }();
+  if ((d + GC_BK - 1) / GC_BK < min_nk) return 1;
   return gc_stages(O, k, E, false, GC_CS) >= 4 ? GC_CS : 1;
 }
 
