@@ -153,7 +153,12 @@ struct Cfg {
   static constexpr int OFF_PREFIX = OFF_SLOT + 16;
   static constexpr int OFF_ROW0 = OFF_PREFIX + (MAX_GROUPS + 1) * 4;
   static constexpr int OFF_SOFF = OFF_ROW0 + (MAX_GROUPS + 1) * 4;
-  static constexpr int OFF_STG = (OFF_SOFF + OFF_INTS * 4 + 127) / 128 * 128;
+  // EPI_REPLICATE with the row-segment epilogue: the tile's destination rows
+  // [row][slot] (-1: no row), written once per tile by the first warp of each
+  // lane quadrant and read by all four
+  static constexpr int DST_BYTES = (EPI == EPI_REPLICATE && ROWSEG) ? BM * 8 * 4 : 0;
+  static constexpr int OFF_DST = OFF_SOFF + OFF_INTS * 4;
+  static constexpr int OFF_STG = (OFF_DST + DST_BYTES + 127) / 128 * 128;
   static constexpr int SMEM = 1024 + OFF_STG + STG_BYTES;
   static_assert(OFF_BARS % 8 == 0 && OFF_STG % 128 == 0, "shared memory alignment");
   static_assert(SMEM <= 232448, "shared memory per CTA");
@@ -179,6 +184,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   int* tile_prefix = reinterpret_cast<int*>(smem + C::OFF_PREFIX);
   int* row0 = reinterpret_cast<int*>(smem + C::OFF_ROW0);
   int* s_off = reinterpret_cast<int*>(smem + C::OFF_SOFF);  // [C::OFF_INTS]
+  int* s_dst = reinterpret_cast<int*>(smem + C::OFF_DST);    // [BM][8] (EPI_REPLICATE, row segments)
   uint8_t* stg_all = smem + C::OFF_STG;                      // epilogue staging
 
   const int warp = threadIdx.x >> 5;
@@ -428,9 +434,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           sc = p.scale[dest];
         }
       }
-      // EPI_REPLICATE: this row's destinations, read once per tile.
+      // EPI_REPLICATE: this row's destinations, read once per tile (with the
+      // row-segment epilogue by the quadrant's first warp only, into s_dst;
+      // the other three read them there after the first slab's barrier, and
+      // the last slab's barrier orders the next tile's writes after every read)
       int rdst[8];
-      if (EPI == EPI_REPLICATE) {
+      if (EPI == EPI_REPLICATE && C::ROWSEG) {
+        if (part == 0) {
+          int* sd = s_dst + row_in_tile * 8;
+#pragma unroll
+          for (int r = 0; r < 8; ++r) {
+            if (r >= p.rep_k) break;
+            int dst = -1;
+            if (valid) {
+              const long long entry = out_row * p.rep_k + r;
+              dst = p.perm[entry];
+              if (p.rep_counts) {
+                dst += s_off[p.rep_idx[entry]];
+                p.rep_perm_out[dst] = static_cast<int32_t>(entry);
+              }
+            }
+            sd[r] = dst;
+          }
+        }
+      } else if (EPI == EPI_REPLICATE) {
 #pragma unroll
         for (int r = 0; r < 8; ++r) {
           rdst[r] = 0;
@@ -500,15 +527,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             __nv_bfloat16* ob = reinterpret_cast<__nv_bfloat16*>(p.out);
             if (EPI == EPI_REPLICATE) {
               // the row's expert-order slots, then (optionally) its own row
+              const int* sd = s_dst + (q * 32 + rr) * 8;  // staged row rr is row q * 32 + rr of the tile
 #pragma unroll
               for (int r = 0; r < 8; ++r) {
                 if (r >= p.rep_k) break;  // uniform across the warp
-                const int dr = __shfl_sync(0xffffffffu, rdst[r], rr);
-                if (rvalid && col < p.N) *reinterpret_cast<U4*>(ob + (long long)dr * p.ldo + col) = q4;
+                const int dr = sd[r];
+                if (rvalid && dr >= 0 && col < p.N) *reinterpret_cast<U4*>(ob + (long long)dr * p.ldo + col) = q4;
               }
-              const long long orow_r = __shfl_sync(0xffffffffu, out_row, rr);
               if (rvalid && col < p.N && p.self_row_base >= 0)
-                *reinterpret_cast<U4*>(ob + (p.self_row_base + orow_r) * p.ldo + col) = q4;
+                *reinterpret_cast<U4*>(ob + (p.self_row_base + out_row - lane + rr) * p.ldo + col) = q4;
             } else {
               const long long drow = __shfl_sync(0xffffffffu, dest, rr);
               if (rvalid && col < p.N) *reinterpret_cast<U4*>(ob + drow * p.ldo + col) = q4;
