@@ -229,6 +229,35 @@ ec2moe_status check_mask(const ec2moe_layer_desc* d, const uint8_t* mask, uint32
 // K range is split so every SM streams, the partial sums (fp32) are reduced,
 // weighted and combined by one small kernel.
 constexpr int SPLITK_MAX = 8;
+
+// Decode steps of at most gate_prefetch_max_tokens() tokens whose up
+// projection runs on the swapped-operand kernel: the small-batch decision
+// kernel prefetches into L2 the first bytes of the weight tile each of that
+// kernel's CTAs streams first (W1, and W3 for SwiGLU), about 80 MB in all,
+// while the codec kernels between them leave HBM idle.
+constexpr long long PREFETCH_BUDGET = 80LL << 20;
+void set_weight_prefetch(const ec2moe_layer_desc* d, const ec2moe_layer_weights* w, int n_allowed, GateArgs* ga) {
+  const long long n = (long long)d->T * d->k;
+  if (d->dtype != EC2MOE_BF16 || !ga->gate_partial || d->T > gate_prefetch_max_tokens() || !swap_gemm_enabled() ||
+      n > SWAP_MAX_ROWS)
+    return;
+  const bool glu = d->act == EC2MOE_SWIGLU;
+  const int tile_rows = glu ? 64 : 128;  // rows of W1 (and W3) per swapped-GEMM weight tile
+  if (d->d_ff % tile_rows != 0) return;
+  const long long experts = n < n_allowed ? n : n_allowed;
+  const long long units = experts * (d->d_ff / tile_rows);
+  const int ctas = static_cast<int>(units < sm_count() ? units : sm_count());
+  const long long per_row = PREFETCH_BUDGET / ((long long)ctas * tile_rows * (glu ? 2 : 1));
+  const long long row_bytes = (long long)d->d * 2;
+  const int bytes = static_cast<int>((per_row < row_bytes ? per_row : row_bytes) / 16 * 16);
+  if (bytes < 16) return;
+  ga->pf_w1 = w->W1;
+  ga->pf_w3 = glu ? w->W3 : nullptr;
+  ga->pf_dff = d->d_ff;
+  ga->pf_tile_rows = tile_rows;
+  ga->pf_units = ctas;
+  ga->pf_row_bytes = bytes;
+}
 bool splitk_possible(const ec2moe_layer_desc* d) {
   const long long n = (long long)d->T * d->k;
   return d->dtype == EC2MOE_BF16 && n >= 1 && n <= 128 && d->d_ff >= 4096 && d->d % 4 == 0;
@@ -787,6 +816,7 @@ ec2moe_status ec2moe_layer_forward(const ec2moe_layer_desc* desc, const ec2moe_l
   }
   if (gate_partial_bytes(desc->T, desc->d, desc->E, desc->n_groups))
     ga.gate_partial = reinterpret_cast<float*>(ws + L.gpart);
+  set_weight_prefetch(desc, w, n_allowed, &ga);
   bool routed = false;
   int gate_sms = 0;
   EC2MOE_CUDA(launch_gate(ga, bf, stream, &routed, &gate_sms));

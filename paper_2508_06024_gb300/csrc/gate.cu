@@ -287,7 +287,8 @@ __global__ void __launch_bounds__(WARPS * 32) gate_topk_kernel(const KParams p) 
 // Same arithmetic as gate_topk_kernel: key = l_i (K = 1) or (m_k - lse_k) + l_i,
 // Top-k by k rounds of a warp argmax with ties to the lower index, weight
 // g_i = exp((m_k - LSE_m) + (l_i - lse_k)).
-__device__ void decide_token_warp(const KParams& p, const float* L, int tok, int lane, int* s_idx) {
+__device__ void decide_token_warp(const KParams& p, const float* L, int tok, int lane, int* s_idx,
+                                  bool write_out = true) {
   const int nglob = (p.K == 1) ? 0 : p.K;
   const int gsize = p.E / p.K;
   float lv[4];
@@ -406,8 +407,10 @@ __device__ void decide_token_warp(const KParams& p, const float* L, int tok, int
     }
   }
   if (lane < p.k) {
-    p.topk_idx[(size_t)tok * p.k + lane] = id_mine;
-    p.topk_w[(size_t)tok * p.k + lane] = p.renorm ? w_mine / wsum : w_mine;
+    if (write_out) {
+      p.topk_idx[(size_t)tok * p.k + lane] = id_mine;
+      p.topk_w[(size_t)tok * p.k + lane] = p.renorm ? w_mine / wsum : w_mine;
+    }
     if (s_idx) s_idx[lane] = id_mine;
   }
 }
@@ -797,6 +800,11 @@ __global__ void __launch_bounds__(GP_THREADS) gate_partial_kernel(const KParams 
 // split four ways (group g adds chunks g, g + 4, ... in order; then the four
 // group sums are added in group order), so each thread keeps eight loads in
 // flight and the result does not depend on the launch.
+// With the prefetch (p.pf_w1, one tile of tokens) every CTA takes the same
+// decisions, CTA 0 alone writes them, and CTA u then prefetches into L2 the
+// first p.pf_row_bytes of each row of weight tile u of the up projection (the
+// first tile the swapped-operand GEMM's CTA u streams), so the HBM otherwise
+// idle during the codec kernels that follow fills L2 with weights.
 constexpr int GD_SPLIT = 4;
 __global__ void __launch_bounds__(SL_THREADS) gate_decide_kernel(const KParams p, const float* __restrict__ part,
                                                                  int n_chunks) {
@@ -807,8 +815,11 @@ __global__ void __launch_bounds__(SL_THREADS) gate_decide_kernel(const KParams p
   float* sGrp = sLog + pairs;                                          // [GD_SPLIT][GD_BT * O]
   int* sIdx = reinterpret_cast<int*>(sGrp + GD_SPLIT * pairs);        // [GD_BT * k]
   __shared__ int s_base[128];
+  __shared__ int s_active[129];  // prefetch: chosen experts in id order, then their count
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int tile = blockIdx.x;
+  const bool pf = p.pf_w1 != nullptr;
+  const int tile = pf ? 0 : blockIdx.x;
+  const bool writer = !pf || blockIdx.x == 0;
   pdl_trigger();
   pdl_wait();
   const size_t plane = (size_t)p.T * O;
@@ -842,16 +853,48 @@ __global__ void __launch_bounds__(SL_THREADS) gate_decide_kernel(const KParams p
   __syncthreads();
   for (int jj = warp; jj < GD_BT; jj += SL_THREADS / 32) {
     const int tok = tile * GD_BT + jj;
-    if (tok < p.T) decide_token_warp(p, sLog + jj * O, tok, lane, p.route_counts ? sIdx + jj * p.k : nullptr);
+    if (tok < p.T)
+      decide_token_warp(p, sLog + jj * O, tok, lane, (p.route_counts || pf) ? sIdx + jj * p.k : nullptr, writer);
   }
   __syncthreads();
-  if (p.route_counts) route_tile(p, tile, GD_BT, sIdx, s_base);
+  if (writer && p.route_counts) route_tile(p, tile, GD_BT, sIdx, s_base);
+  if (!pf) return;
+  // the chosen experts in id order (the swapped GEMM's active groups)
+  if (warp == 0) {
+    const int n_ent = p.T * p.k;
+    int count = 0;
+    for (int e0 = 0; e0 < p.E; e0 += 32) {
+      const int e = e0 + lane;
+      bool hit = false;
+      for (int i = 0; i < n_ent; ++i) hit |= (sIdx[i] == e);
+      const unsigned m = __ballot_sync(0xffffffffu, hit && e < p.E);
+      if (hit && e < p.E) s_active[count + __popc(m & ((1u << lane) - 1u))] = e;
+      count += __popc(m);
+    }
+    if (lane == 0) s_active[128] = count;
+  }
+  __syncthreads();
+  const int tiles_per_expert = p.pf_dff / p.pf_tile_rows;
+  const int a = blockIdx.x / tiles_per_expert;
+  if (a >= s_active[128]) return;
+  const int e = s_active[a];
+  const int nb = blockIdx.x % tiles_per_expert;
+  const int n_mats = p.pf_w3 ? 2 : 1;
+  if (threadIdx.x < n_mats * p.pf_tile_rows) {
+    const int m = threadIdx.x / p.pf_tile_rows;
+    const long long row = (long long)e * p.pf_dff + (long long)nb * p.pf_tile_rows + threadIdx.x % p.pf_tile_rows;
+    const char* base = static_cast<const char*>(m ? p.pf_w3 : p.pf_w1);
+    const char* src = base + row * (long long)p.d * 2;
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src), "r"(p.pf_row_bytes) : "memory");
+  }
 }
 
 constexpr int GP_MAX_T = 256;
 constexpr int GP_MIN_D = 1024;
 
 }  // namespace
+
+int gate_prefetch_max_tokens() { return GD_BT; }
 
 size_t gate_partial_bytes(int T, int d, int E, int K) {
   const int O = E + (K == 1 ? 0 : K);
@@ -877,7 +920,9 @@ cudaError_t launch_gate_partial(const GateArgs& a, const KParams& p, int O, cuda
   e = ensure_smem_attr(reinterpret_cast<const void*>(gate_decide_kernel), smem_b);
   if (e != cudaSuccess) return e;
   KernelScope ks("gate_decide", s);
-  e = launch_kernel(gate_decide_kernel, dim3((a.T + GD_BT - 1) / GD_BT), dim3(SL_THREADS), (size_t)smem_b, s, p,
+  // with the prefetch: one CTA per swapped-GEMM CTA, all on the one tile
+  const int blocks = p.pf_w1 ? a.pf_units : (a.T + GD_BT - 1) / GD_BT;
+  e = launch_kernel(gate_decide_kernel, dim3(blocks), dim3(SL_THREADS), (size_t)smem_b, s, p,
                     static_cast<const float*>(a.gate_partial), n_chunks);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
@@ -908,6 +953,9 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* rout
   p.topk_w = a.topk_w;
   p.route_counts = nullptr;
   p.route_rel = nullptr;
+  p.pf_w1 = nullptr;
+  p.pf_w3 = nullptr;
+  p.pf_dff = p.pf_tile_rows = p.pf_row_bytes = 0;
   const int O = a.E + (a.K == 1 ? 0 : a.K);
   cudaError_t e;
   if (a.gate_partial && gate_partial_bytes(a.T, a.d, a.E, a.K) &&
@@ -917,6 +965,18 @@ cudaError_t launch_gate(const GateArgs& a, bool bf16, cudaStream_t s, bool* rout
       p.route_counts = a.route_counts;
       p.route_rel = a.route_rel;
       if (routed) *routed = true;
+    }
+    // the weight prefetch needs one tile of tokens, whole 16-byte pieces
+    // and tiles that divide d_ff
+    if (a.pf_w1 && a.T <= GD_BT && a.pf_units > 0 && a.pf_tile_rows > 0 && a.pf_tile_rows <= 128 &&
+        a.pf_dff % a.pf_tile_rows == 0 && a.pf_row_bytes >= 16 && a.pf_row_bytes % 16 == 0 &&
+        a.pf_row_bytes <= a.d * 2 && reinterpret_cast<uintptr_t>(a.pf_w1) % 16 == 0 &&
+        reinterpret_cast<uintptr_t>(a.pf_w3) % 16 == 0 && a.d % 8 == 0) {
+      p.pf_w1 = a.pf_w1;
+      p.pf_w3 = a.pf_w3;
+      p.pf_dff = a.pf_dff;
+      p.pf_tile_rows = a.pf_tile_rows;
+      p.pf_row_bytes = a.pf_row_bytes;
     }
     if (held_sms) *held_sms = (a.T + GD_BT - 1) / GD_BT;
     return bf16 ? launch_gate_partial<__nv_bfloat16>(a, p, O, s) : launch_gate_partial<float>(a, p, O, s);

@@ -26,6 +26,11 @@ struct KParams {
   float* topk_w;
   int32_t* route_counts;  // fused routing: per-expert row counters (zero at launch); nullptr = gate only
   int32_t* route_rel;     // fused routing: [T*k] row of each entry relative to its expert's first row
+  // L2 prefetch of the decode up projection's first weight tiles by the
+  // small-batch decision kernel (GateArgs::pf_*); pf_w1 == nullptr: none
+  const void* pf_w1;
+  const void* pf_w3;
+  int pf_dff, pf_tile_rows, pf_row_bytes;
 };
 
 // Tensor-core gate (bf16, at most 80 gate rows) with its prep kernel; sets

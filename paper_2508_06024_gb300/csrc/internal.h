@@ -88,7 +88,20 @@ struct GateArgs {
   // batches then split d_model across CTAs (partial logits, then a decision
   // kernel); nullptr: the per-tile gates.
   float* gate_partial;
+  // Optional, with gate_partial and T <= gate_prefetch_max_tokens(): once the
+  // decision kernel knows the chosen experts, pf_units of its CTAs each
+  // prefetch into L2 the first pf_row_bytes of every weight row of one
+  // weight tile of the decode up projection, in the order the swapped-operand
+  // GEMM's CTAs take their first tiles (launch_gemm_swap: CTA u starts with
+  // unit u = (chosen expert u / (d_ff / pf_tile_rows) in id order, tile u mod
+  // that), pf_tile_rows rows of W1 and, for SwiGLU, the same rows of W3).
+  // Results do not depend on it.  pf_w1 == nullptr: no prefetch.
+  const void* pf_w1;  // [E, d_ff, d] bf16
+  const void* pf_w3;  // [E, d_ff, d] bf16, or nullptr (GELU)
+  int pf_dff, pf_tile_rows, pf_units, pf_row_bytes;
 };
+// Largest batch whose decision kernel can prefetch the up projection's weights.
+int gate_prefetch_max_tokens();
 // Bytes of the prepared split gate rows (0 when the tensor-core gate does not apply).
 size_t gate_split_bytes(int E, int K, int d, bool bf16);
 // Bytes of the small-batch gate's partial logits (0 when that gate does not apply).

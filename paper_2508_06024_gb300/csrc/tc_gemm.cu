@@ -36,6 +36,13 @@
 // a cluster barrier precedes its release.  After an abort the odd CTA cannot
 // observe its own copies, so it waits a fixed, bounded time for them to land.
 //
+// Two pairs per cluster (QUAD, opt-in): four CTAs, pair p = CTAs 2p and
+// 2p + 1, both pairs on the same 256 rows of A and on N tiles 2j and 2j + 1.
+// Each CTA loads 64 of its 128 A rows and multicasts them to the CTA of the
+// same pair rank in the other pair; a destination's bytes complete on the full
+// barrier of its own pair's even CTA.  Stage-freeing commits go to all four
+// CTAs and each empty barrier counts both pairs' commits.
+//
 // Every mbarrier wait is bounded by a clock64 budget.  A wait that gives up
 // sets the device error word, raises a CTA-wide abort flag that ends every
 // other wait at once, waits (again bounded) for the CTA's own TMA copies and
@@ -164,10 +171,11 @@ struct Cfg {
   static_assert(SMEM <= 232448, "shared memory per CTA");
 };
 
-template <int BN, int EPI, int STAGES, bool PAIR>
+template <int BN, int EPI, int STAGES, bool PAIR, bool QUAD = false>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     tc_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmB2, const Params p) {
+  static_assert(!QUAD || PAIR, "two pairs per cluster need CTA pairs");
   using C = Cfg<BN, EPI, STAGES, PAIR>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -189,8 +197,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // PAIR: rank in the CTA pair (0 issues the MMAs), the pair's tile stream
-  const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+  // PAIR: rank in the CTA pair (0 issues the MMAs), the pair's even CTA in
+  // the cluster, the cluster's tile stream.  QUAD: the cluster holds two pairs
+  // (CTAs 0-1 and 2-3) on the same 256 rows of A and neighbouring N tiles;
+  // each CTA loads half of its 128 A rows and multicasts them to the CTA of
+  // the same pair rank in the other pair.
+  const uint32_t crank = PAIR ? cluster_ctarank() : 0u;
+  const uint32_t rank = crank & 1u;
+  const uint32_t leader = crank & ~1u;
+  const int pp = QUAD ? static_cast<int>(crank >> 1) : 0;
+  const int ntn = QUAD ? p.n_tiles_n / 2 : p.n_tiles_n;  // N tiles of a cluster tile's stream
   const int tile_first = PAIR ? static_cast<int>(cluster_id_x()) : static_cast<int>(blockIdx.x);
   const int tile_step = PAIR ? static_cast<int>(cluster_count_x()) : static_cast<int>(gridDim.x);
   // Barrier set-up, TMEM allocation and descriptor prefetch overlap the
@@ -200,7 +216,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), 1);
+      // QUAD: a stage is free once both pairs' MMAs have read it (the other
+      // pair multicasts into it)
+      mbar_init(smem_u32(&empty[s]), QUAD ? 2 : 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(smem_u32(&tfull[a]), 1);
@@ -264,7 +282,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   const uint32_t tmem_base = *tmem_slot;
   // Split-K (EPI_PARTIAL): tile t covers output tile t / split_k and the
   // k-blocks [ks * kb_per_split, ...) with ks = t % split_k.
-  const int n_tiles = tile_prefix[p.G] * p.n_tiles_n * p.split_k;
+  const int n_tiles = tile_prefix[p.G] * ntn * p.split_k;
   const int num_kb = (p.K + BK - 1) / BK;
   const long long budget = p.timeout;
 
@@ -278,10 +296,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int cursor = 0;
       bool ok = true;
       for (int tile = tile_first; tile < n_tiles && ok; tile += tile_step) {
-        const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
+        const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, ntn, cursor);
+        const int n_blk = QUAD ? 2 * tc.n_blk + pp : tc.n_blk;
         const int a_row = static_cast<int>(p.a_row_base) + (p.offsets ? row0[tc.g] : (p.a_shared ? 0 : row0[tc.g])) +
                           tc.m_blk * C::TILE_M + static_cast<int>(rank) * BM;
-        const int b_row = tc.g * p.b_group_rows + tc.n_blk * C::BN_OUT;
+        const int b_row = tc.g * p.b_group_rows + n_blk * C::BN_OUT;
         const int kb0 = (tile % p.split_k) * p.kb_per_split;
         const int kb1 = kb0 + p.kb_per_split < num_kb ? kb0 + p.kb_per_split : num_kb;
         for (int kb = kb0; kb < kb1; ++kb) {
@@ -293,8 +312,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (PAIR) {
             // both halves complete on the even CTA's full barrier
             if (rank == 0) mbar_expect_tx(fb, 2 * C::STAGE_BYTES);
-            const uint32_t fb0 = rank == 0 ? fb : map_to_rank(fb, 0);
-            tma_load_2d_to_pair_bar(smem_u32(sA + stage * C::A_BYTES), &tmA, kb * BK, a_row, fb0);
+            const uint32_t fb0 = rank == 0 ? fb : map_to_rank(fb, leader);
+            if (QUAD) {
+              // rows [pp * 64, pp * 64 + 64) of this CTA's 128, to both pairs
+              tma_load_2d_mc_pair(smem_u32(sA + stage * C::A_BYTES + pp * (BM / 2) * BK * 2), &tmA, kb * BK,
+                                  a_row + pp * (BM / 2), fb0, static_cast<uint16_t>(0x5u << rank));
+            } else {
+              tma_load_2d_to_pair_bar(smem_u32(sA + stage * C::A_BYTES), &tmA, kb * BK, a_row, fb0);
+            }
             // SwiGLU: the even CTA stages the W1 rows of the tile, the odd CTA the W3 rows
             const CUtensorMap* tb = (EPI == EPI_SWIGLU && rank) ? &tmB2 : &tmB;
             tma_load_2d_to_pair_bar(smem_u32(sB + stage * C::B_BYTES), tb, kb * BK,
@@ -349,7 +374,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int cursor = 0;
       bool ok = true, any = false;
       for (int tile = tile_first; tile < n_tiles && ok; tile += tile_step, ++it) {
-        (void)decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
+        (void)decode_tile(tile / p.split_k, tile_prefix, ntn, cursor);
         const int kb0 = (tile % p.split_k) * p.kb_per_split;
         const int kb1 = kb0 + p.kb_per_split < num_kb ? kb0 + p.kb_per_split : num_kb;
         const int acc = it & 1;
@@ -385,7 +410,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int kk = 1; kk < BK / UK; ++kk) umma_bf16(d_tmem, da + 2 * kk, db + 2 * kk, IDESC, 1u);
           }
           any = true;
-          if (PAIR) umma_commit_pair_mc(empty0 + 8u * stage);
+          // QUAD: both pairs' producers wait for this stage
+          if (PAIR) umma_commit_pair_mc(empty0 + 8u * stage, QUAD ? 0xF : 0x3);
           else umma_commit(empty0 + 8u * stage);
           if (++stage == STAGES) {
             stage = 0;
@@ -393,7 +419,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
         }
         if (!ok) break;
-        if (PAIR) umma_commit_pair_mc(smem_u32(&tfull[acc]));
+        if (PAIR) umma_commit_pair_mc(smem_u32(&tfull[acc]), static_cast<uint16_t>(0x3u << leader));
         else umma_commit(smem_u32(&tfull[acc]));
       }
       if ((!ok || *abort_flag) && any) {
@@ -411,7 +437,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     int it = 0;
     int cursor = 0;
     for (int tile = tile_first; tile < n_tiles; tile += tile_step, ++it) {
-      const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, p.n_tiles_n, cursor);
+      const TileCoord tc = decode_tile(tile / p.split_k, tile_prefix, ntn, cursor);
+      const int n_blk = QUAD ? 2 * tc.n_blk + pp : tc.n_blk;
       const int ks = tile % p.split_k;
       (void)ks;
       const int acc = it & 1;
@@ -518,7 +545,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           asm volatile("bar.sync %0, 128;" ::"r"(1 + q) : "memory");
           const int seg = lane & 7;
-          const int col = tc.n_blk * C::BN_OUT + sl * C::SLAB + seg * 8;
+          const int col = n_blk * C::BN_OUT + sl * C::SLAB + seg * 8;
 #pragma unroll
           for (int pass = 0; pass < 2; ++pass) {
             const int rr = part * 8 + pass * 4 + (lane >> 3);
@@ -547,7 +574,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         __syncwarp();
         if (lane == 0) {
           // PAIR: both CTAs release the accumulator on the even CTA's barrier
-          if (PAIR) mbar_arrive_remote(map_to_rank(smem_u32(&tempty[acc]), 0));
+          if (PAIR) mbar_arrive_remote(map_to_rank(smem_u32(&tempty[acc]), leader));
           else mbar_arrive(smem_u32(&tempty[acc]));
         }
         continue;
@@ -577,7 +604,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           }
           tmem_wait();
         }
-        const int col = tc.n_blk * C::BN_OUT + c0;
+        const int col = n_blk * C::BN_OUT + c0;
         float v[C::CW];
 #pragma unroll
         for (int i = 0; i < C::CW; ++i) v[i] = __uint_as_float(slot ? rv[1][i] : rv[0][i]);
@@ -635,7 +662,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       tc_fence_before();
       __syncwarp();
       if (lane == 0) {
-        if (PAIR) mbar_arrive_remote(map_to_rank(smem_u32(&tempty[acc]), 0));
+        if (PAIR) mbar_arrive_remote(map_to_rank(smem_u32(&tempty[acc]), leader));
         else mbar_arrive(smem_u32(&tempty[acc]));
       }
     }
@@ -749,9 +776,9 @@ const char* kernel_name(int epi) {
   }
 }
 
-// Clusters of two CTAs of `kernel` that fit on the device at once (cached per
-// device and kernel); 0 when the query fails.
-int max_pair_clusters(const void* kernel, int smem) {
+// Clusters of `cdim` CTAs (2: one pair, 4: two pairs) of `kernel` that fit on
+// the device at once (cached per device and kernel); 0 when the query fails.
+int max_pair_clusters(const void* kernel, int smem, int cdim) {
   struct Entry {
     int dev;
     const void* kernel;
@@ -766,12 +793,12 @@ int max_pair_clusters(const void* kernel, int smem) {
   for (int i = 0; i < used; ++i)
     if (cache[i].dev == dev && cache[i].kernel == kernel) return cache[i].n;
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(2 * sm_count());
+  cfg.gridDim = dim3(cdim * sm_count());
   cfg.blockDim = dim3(NUM_THREADS);
   cfg.dynamicSmemBytes = smem;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.x = cdim;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
@@ -786,15 +813,16 @@ int max_pair_clusters(const void* kernel, int smem) {
 }
 
 template <typename... KArgs, typename... Args>
-cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, size_t smem, cudaStream_t s, Args&&... args) {
+cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, int cdim, size_t smem, cudaStream_t s,
+                         Args&&... args) {
   cudaLaunchConfig_t cfg{};
-  cfg.gridDim = dim3(2 * clusters);
+  cfg.gridDim = dim3(cdim * clusters);
   cfg.blockDim = dim3(NUM_THREADS);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.x = cdim;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -804,15 +832,15 @@ cudaError_t launch_pairs(void (*kernel)(KArgs...), int clusters, size_t smem, cu
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
-template <int BN, int EPI, int STAGES, bool PAIR = false>
+template <int BN, int EPI, int STAGES, bool PAIR = false, bool QUAD = false>
 cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   using C = Cfg<BN, EPI, STAGES, PAIR>;
-  const void* kfn = reinterpret_cast<const void*>(tc_gemm_kernel<BN, EPI, STAGES, PAIR>);
+  const void* kfn = reinterpret_cast<const void*>(tc_gemm_kernel<BN, EPI, STAGES, PAIR, QUAD>);
   cudaError_t attr_err = ensure_smem_attr(kfn, C::SMEM);
   if (attr_err != cudaSuccess) return attr_err;
   CUtensorMap mA, mB, mB2;
   const int b_box = (EPI == EPI_SWIGLU || PAIR) ? BN / 2 : BN;
-  if (!make_map(&mA, a.A, a.a_rows, a.K, BM)) return cudaErrorInvalidValue;
+  if (!make_map(&mA, a.A, a.a_rows, a.K, QUAD ? BM / 2 : BM)) return cudaErrorInvalidValue;
   if (!make_map(&mB, a.B, a.b_rows, a.K, b_box)) return cudaErrorInvalidValue;
   if (EPI == EPI_SWIGLU) {
     if (!make_map(&mB2, a.B2, a.b_rows, a.K, b_box)) return cudaErrorInvalidValue;
@@ -854,11 +882,15 @@ cudaError_t launch_cfg(const GemmArgs& a, cudaStream_t s) {
   const long long m_tiles_max = a.max_rows / C::TILE_M + a.G;
   long long tiles = m_tiles_max * p.n_tiles_n * p.split_k;
   if (PAIR) {
-    int clusters = max_pair_clusters(kfn, C::SMEM);
+    // QUAD: a cluster tile is two N tiles (p.n_tiles_n is even)
+    if (QUAD) tiles /= 2;
+    const int cdim = QUAD ? 4 : 2;
+    int clusters = max_pair_clusters(kfn, C::SMEM, cdim);
     if (clusters < 1) return cudaErrorInvalidConfiguration;
     if (tiles < clusters) clusters = static_cast<int>(tiles < 1 ? 1 : tiles);
     KernelScope ks(a.name ? a.name : kernel_name(EPI), s);
-    cudaError_t le = launch_pairs(tc_gemm_kernel<BN, EPI, STAGES, PAIR>, clusters, (size_t)C::SMEM, s, mA, mB, mB2, p);
+    cudaError_t le = launch_pairs(tc_gemm_kernel<BN, EPI, STAGES, PAIR, QUAD>, clusters, cdim, (size_t)C::SMEM, s, mA,
+                                  mB, mB2, p);
     if (le != cudaSuccess) return le;
     return cudaGetLastError();
   }
@@ -878,10 +910,11 @@ constexpr int stages_for(int b_rows) {
 }
 
 template <int EPI>
-cudaError_t launch_epi(const GemmArgs& a, int bn, bool pair, cudaStream_t s) {
+cudaError_t launch_epi(const GemmArgs& a, int bn, bool pair, bool quad, cudaStream_t s) {
   if (pair) {
     if constexpr (EPI == EPI_STORE || EPI == EPI_GELU || EPI == EPI_SWIGLU || EPI == EPI_SCATTER ||
                   EPI == EPI_REPLICATE) {
+      if (bn == 256 && quad) return launch_cfg<256, EPI, stages_for(128), true, true>(a, s);
       if (bn == 256) return launch_cfg<256, EPI, stages_for(128), true>(a, s);
       if (bn == 128) return launch_cfg<128, EPI, stages_for(64), true>(a, s);
     }
@@ -964,6 +997,23 @@ bool use_pairs(const GemmArgs& a, int epi) {
   return pad2 <= 1.1 * pad1;
 }
 
+// Whether a pair GEMM runs two pairs per cluster on neighbouring N tiles of
+// the same rows, each CTA loading half of its A rows and multicasting them to
+// the other pair (QUAD): 256-column tiles and an even N-tile count.
+// EC2MOE_GEMM_QUAD=0 / =1 in the environment forbids / allows it (A/B
+// comparisons; both compute the same result).
+bool use_quad(const GemmArgs& a, int epi, int bn) {
+  // 0: never; 1: every eligible GEMM; 2: the scattering (down) projections only
+  static const int allowed = [] {
+    const char* v = getenv("EC2MOE_GEMM_QUAD");
+    return v ? (v[0] == '1' ? 1 : (v[0] == 'd' ? 2 : 0)) : 0;
+  }();
+  if (!allowed || bn != 256 || (allowed == 2 && epi != EPI_SCATTER)) return false;
+  const int bn_out = epi == EPI_SWIGLU ? bn / 2 : bn;
+  const int n_tiles_n = (a.N + bn_out - 1) / bn_out;
+  return n_tiles_n % 2 == 0;
+}
+
 cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
   if (a.G < 1 || a.G > MAX_GROUPS || a.N % 32 != 0 || a.K % 8 != 0) return cudaErrorInvalidValue;
   bool pair = use_pairs(a, epi);
@@ -973,12 +1023,13 @@ cudaError_t launch_gemm_tc(const GemmArgs& a, int epi, cudaStream_t s) {
     pair = false;
     bn = choose_bn(a, epi, false);
   }
+  const bool quad = pair && use_quad(a, epi, bn);
   switch (epi) {
-    case EPI_STORE: return launch_epi<EPI_STORE>(a, bn, pair, s);
-    case EPI_GELU: return launch_epi<EPI_GELU>(a, bn, pair, s);
-    case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, pair, s);
-    case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, pair, s);
-    case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, pair, s);
+    case EPI_STORE: return launch_epi<EPI_STORE>(a, bn, pair, quad, s);
+    case EPI_GELU: return launch_epi<EPI_GELU>(a, bn, pair, quad, s);
+    case EPI_SWIGLU: return launch_epi<EPI_SWIGLU>(a, bn, pair, quad, s);
+    case EPI_SCATTER: return launch_epi<EPI_SCATTER>(a, bn, pair, quad, s);
+    case EPI_REPLICATE: return launch_epi<EPI_REPLICATE>(a, bn, pair, quad, s);
     case EPI_PARTIAL:
       if (!a.partial || a.N % 4 != 0) return cudaErrorInvalidValue;
       return bn >= 256 ? launch_cfg<256, EPI_PARTIAL, stages_for(256)>(a, s)

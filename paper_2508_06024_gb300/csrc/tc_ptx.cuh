@@ -81,6 +81,18 @@ __device__ __forceinline__ void tma_load_2d_to_pair_bar(uint32_t dst, const CUte
       "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
       : "memory");
 }
+// The same copy multicast to the CTAs of `cta_mask` (same shared offset in
+// each); each destination's bytes complete on the mbarrier at `bar`'s offset
+// in the even CTA of that destination's pair (`bar` names the issuing CTA's
+// pair leader).
+__device__ __forceinline__ void tma_load_2d_mc_pair(uint32_t dst, const CUtensorMap* tm, int x, int y, uint32_t bar,
+                                                    uint16_t cta_mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster.cta_group::"
+      "2 [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar), "h"(cta_mask)
+      : "memory");
+}
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* tm) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tm)) : "memory");
 }
@@ -272,12 +284,13 @@ __device__ __forceinline__ void umma_bf16_pair(uint32_t d_tmem, uint64_t da, uin
       "l"(da), "l"(db), "r"(idesc), "r"(accum)
       : "memory");
 }
-// Arrive on the barrier at shared address `bar` in both CTAs of the pair once
-// the pair MMAs issued so far have completed.
-__device__ __forceinline__ void umma_commit_pair_mc(uint32_t bar) {
+// Arrive on the barrier at shared address `bar` in the CTAs of `cta_mask`
+// (both CTAs of the pair: 3; with two pairs per cluster also the other pair's)
+// once the pair MMAs issued so far have completed.
+__device__ __forceinline__ void umma_commit_pair_mc(uint32_t bar, uint16_t cta_mask = 3) {
   asm volatile(
       "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
-      "h"(static_cast<uint16_t>(3))
+      "h"(cta_mask)
       : "memory");
 }
 // Arrive on the issuing CTA's own barrier once its pair MMAs have completed.
