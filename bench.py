@@ -681,6 +681,7 @@ def run_ours(args):
                 "ms_per_step": round(t_e2e, 5),
                 "serial_value": round(whole_job_tokens_per_s(world, cfg.T, t_serial), 1),
                 "serial_ms_per_step": round(t_serial, 5)},
+        "expert_histogram": [int(c) for c in run.counts.cpu().tolist()],
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
         "peaks": {"source": peaks_src, "hbm_gbs": peaks["hbm_gbs"], "bf16_tflops": peaks["bf16_tflops"]},

@@ -354,6 +354,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           for (int s = 0; s < STAGES; ++s)
             if (issued & (1u << s)) mbar_drain(smem_u32(&full[s]), (issued_phase >> s) & 1u, DRAIN_CYCLES);
         }
+        if (QUAD) {
+          // the other pair's multicasts into this CTA's stages are not all
+          // counted on barriers this CTA waited on: a fixed time to land too
+          const unsigned long long t0 = globaltimer_ns();
+          while (globaltimer_ns() - t0 < 200000ull) __nanosleep(1000);
+        }
       }
     }
   } else if (warp == 1) {

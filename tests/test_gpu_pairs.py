@@ -38,3 +38,15 @@ def test_layer_parity_with_pair_gemm_setting(mode):
                         os.path.join(ROOT, "tests", "test_gpu_parity.py"), "-k", SELECT],
                        cwd=ROOT, env=env, capture_output=True, text=True, timeout=1500)
     assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-2000:]
+
+
+def test_zero_wait_budget_on_two_pair_clusters():
+    """A timeout inside the two-pair cluster GEMM (every wait given a zero
+    budget) ends with EC2MOE_ERR_TIMEOUT and a context that still runs the
+    layer to the same output, as for the other kernel families."""
+    env = dict(os.environ, EC2MOE_GEMM_QUAD="1")
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-m", "gpu", "-p", "no:cacheprovider",
+                        os.path.join(ROOT, "tests", "test_gpu_failure.py"), "-k", "mixtral-pairs"],
+                       cwd=ROOT, env=env, capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-2000:]
+
