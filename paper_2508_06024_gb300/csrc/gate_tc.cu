@@ -57,9 +57,9 @@ namespace {
 // memory, counted on the owner's receive barrier), and the owner adds the
 // cluster's partials in CTA order before the bias and the decision; every CTA
 // reserves the rows it decided.  One tile per cluster: such grids are one
-// cluster per tile, run in waves when they exceed the SMs.  A tile's reading
-// of X is then spread over twice the SMs (the per-SM copy rate, not HBM,
-// bounds a 128-token tile's stream).
+// cluster per tile, run in waves when they exceed the SMs.  A tile's stages
+// (the stream of X, the MMAs and the accumulator drains) are then spread over
+// twice the SMs.
 // Every mbarrier wait is bounded; on a timeout the error word is set, copies
 // and MMAs in flight are drained and the CTA finishes its tiles without
 // waiting (the decisions then see garbage logits but still name valid experts).
