@@ -647,6 +647,9 @@ def run_ours(args):
             kern[n]["vs_stream"] = round(sm / kern[n]["avg_ms"], 3)
     if "stream_ms" in kern[dominant]:
         roof["stream_ms"] = kern[dominant]["stream_ms"]
+    # the same bracket around a launch that reads 64 KB: what the one-launch
+    # timing charges every kernel whatever it does
+    floor_ms = stream_reference_ms(torch, dev, stream, flush, 65536, prof_steps)
 
     cpu = None
     if not args.no_cpu_baseline and world == 1:
@@ -669,7 +672,8 @@ def run_ours(args):
                    "kernel_timing": "per launch index, a graph of the whole call with only that launch bracketed "
                                     "by CUDA events, L2 flushed; share = kernel time / step time; stream_ms = one "
                                     "torch launch reading the kernel's algorithmic bytes, bracketed the same way "
-                                    "(HBM-bound kernels); vs_stream = stream_ms / avg_ms"},
+                                    "(HBM-bound kernels); vs_stream = stream_ms / avg_ms",
+                   "timing_floor_ms": round(floor_ms, 5)},
         "layer_tflops": round(layer_flops / (t_step * 1e-3) / 1e12, 2),
         "layer_frac_bf16_peak": round(layer_flops / (t_step * 1e-3) / 1e12 / peaks["bf16_tflops"], 4),
         "roofline": roof,
