@@ -219,6 +219,55 @@ def m_pruning_ignored(l, m, allowed, K, G):
     return g, log_g, np.full(l.shape[0], np.inf)
 
 
+def m_group_factor_dropped(l, m, allowed, K):
+    # Eq. 7 without the group probability: g = p_local
+    g, log_g = _group_gate(l, m, allowed, K)
+    if K == 1 or m is None:
+        return g, log_g
+    b = orc.group_bounds(l.shape[1], K)
+    gof = np.repeat(np.arange(K), np.diff(b))
+    live = np.array([allowed[b[i]:b[i + 1]].any() for i in range(K)])
+    p_group = _masked_softmax(m, live)
+    with np.errstate(divide="ignore", invalid="ignore"):
+        g2 = np.where(allowed[None, :], g / p_group[:, gof], 0.0)
+        log_g2 = np.where(allowed[None, :], log_g - np.log(p_group[:, gof]), -np.inf)
+    return g2, log_g2
+
+
+def m_global_from_local_rows(X, Wl, bl, Wg=None, bg=None):
+    # Eq. 6 evaluated with the first K local gate rows instead of W_global
+    if Wg is None:
+        return _gate_logits(X, Wl, bl, Wg, bg)
+    K = np.asarray(Wg).shape[0]
+    return _gate_logits(X, Wl, bl, np.asarray(Wl)[:K], bg)
+
+
+def m_perm_slot_major(idx, E):
+    # rows of one expert ordered by (slot, token) instead of (token, slot)
+    counts, offsets, _ = _route_tables(idx, E)
+    idx = np.asarray(idx)
+    T, k = idx.shape
+    flat = idx.reshape(-1)
+    t = np.arange(T * k) // k
+    s = np.arange(T * k) % k
+    perm = np.lexsort((t, s, flat)).astype(np.int64)
+    return counts, offsets, perm
+
+
+def m_shared_scaled_by_gate(inp, n_groups, k, act, renorm=False, rows=None, top_groups=0):
+    # the always-on shared experts weighted by the first slot's gate weight
+    out = _layer_forward(inp, n_groups, k, act, renorm, rows, top_groups)
+    if inp.get("W1s") is None:
+        return out
+    X_hat = out["X_hat"]
+    w0 = out["w"][out["rows"], 0][:, None]
+    for s in range(inp["W1s"].shape[0]):
+        W3s = None if inp.get("W3s") is None else inp["W3s"][s]
+        o = orc.expert_ffn(X_hat, inp["W1s"][s], inp["W2s"][s], W3s, act)
+        out["y"] = out["y"] + (w0 - 1.0) * o
+    return out
+
+
 def m_gap_wrong_sign(log_g, idx, allowed):
     b, a = _topk_gaps(log_g, idx, allowed)
     return -b, a
@@ -251,6 +300,10 @@ MUTANTS = [
     ("group_gate_pruned", m_pruned_by_best_local),
     ("group_gate_pruned", m_pruning_ignored),
     ("topk_gaps", m_gap_wrong_sign),
+    ("group_gate", m_group_factor_dropped),
+    ("gate_logits", m_global_from_local_rows),
+    ("route_tables", m_perm_slot_major),
+    ("layer_forward", m_shared_scaled_by_gate),
 ]
 
 
